@@ -30,8 +30,8 @@ log_ndtr (library primitives).
 
 Readings where the paper is silent (identical on the CUDA side):
   * one coin per (chain, step) from Philox stream 0, drawn for every step;
-  * the bisection stops when the bracket is narrower than ``xtol`` (the paper's
-    |Psi(mid) - w| <= tol with tol -> 0); no 3/4-iteration caps;
+  * the bisection stops when the bracket is narrower than ``xtol * max(1, |mid|)``
+    (the paper's |Psi(mid) - w| <= tol with tol -> 0); no 3/4-iteration caps;
   * degenerate h_j: alpha_j = 1 -> 1; alpha_j = 0 or |Delta_{j+1}| = 0 (alpha_j < 1) -> 0;
   * |Delta_tau| = 0 at the residual (probability zero): Y = m^q + sigma G, status bit 1;
   * full accept without a bonus mean returns the last draft row; with one,
@@ -187,7 +187,9 @@ def usample_bisection(D, log_alpha, w, tol=0.0, xtol=1e-12):
 
     Bounds (a+ - 1, a+); while Psi(lower) > w the lower bound becomes
     upper - 2 (upper - lower); then bisection on the sign of Psi(mid) - w until
-    |Psi(mid) - w| <= tol or the bracket is narrower than xtol.
+    |Psi(mid) - w| <= tol or the bracket is narrower than xtol * max(1, |mid|)
+    (the paper leaves tol unspecified; a relative width keeps the loop finite
+    where the fp64 spacing of |mid| exceeds xtol).
     """
     D = np.atleast_1d(np.asarray(D, dtype=np.float64))
     la = np.atleast_1d(np.asarray(log_alpha, dtype=np.float64))
@@ -202,7 +204,7 @@ def usample_bisection(D, log_alpha, w, tol=0.0, xtol=1e-12):
     active = np.ones(D.shape, dtype=bool)
     while True:
         p = psi_cdf(mid, D, la)
-        active &= ~((np.abs(p - w) <= tol) | ((hi - lo) <= xtol))
+        active &= ~((np.abs(p - w) <= tol) | ((hi - lo) <= xtol * np.maximum(1.0, np.abs(mid))))
         if not np.any(active):
             break
         lo = np.where(active & (p < w), mid, lo)

@@ -1,0 +1,384 @@
+"""Benchmark of the speculative-diffusion verification step on GB300.
+
+One step = one sdv_verify call (log-ratio pass, acceptance scan + residual
+U-draw, residual write) on one batch of the pixel-scale workload (B=256 chains,
+L=8 draft steps, d=3x32x32 fp32, block verification) with inputs resident in
+HBM.  Eight input sets (8 x 75.5 MB, well above the 129 MB L2) rotate between
+steps, so every step reads its inputs from HBM.  Steps are captured into CUDA
+graphs and replayed.
+
+Prints ONE JSON line (rank 0):
+  value      verified draft-steps/s (B*L per step), whole job
+  roofline   the log-ratio pass (dominant kernel): algorithmic bytes / its mean
+             duration from CUDA events inside the timed region, vs measured HBM peak
+  e2e        the same metric through the public API from pinned host buffers
+             (host->device copy of the window, device->host copy of results)
+  cpu_baseline  the CPU oracle on a bounded sample of the same workload
+
+--impl reference times the CPU oracle alone (the reference arm of this build).
+"""
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workloads as W  # noqa: E402
+
+METRIC = "verified draft-steps/s and HBM GB/s vs ~8 TB/s; mean accepted steps/target call"
+UNIT = "draft-steps/s"
+N_SETS = 8
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20000)
+    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="pixel", choices=["pixel", "latent", "highres"])
+    p.add_argument("--mode", default="block", choices=["block", "sample"])
+    p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--skip-cpu", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def profile_traffic(kernel_src):
+    """dram bytes per launch of the log-ratio pass from the committed ncu summary, if the
+    kernel source is unchanged since the capture (else None)."""
+    path = os.path.join(ROOT, "profiles", "ratio_partials_pixel.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    h = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt)
+    if not m or not h:
+        return None
+    digest = hashlib.sha256(open(kernel_src, "rb").read()).hexdigest()
+    return float(m.group(1)) if h.group(1) == digest else None
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = [r.split(",") for r in out.strip().splitlines() if r.strip()]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.strip().lower() in ("active", "1", "yes"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def cpu_oracle_rate(inp, seed, mode, seconds, max_chains=None):
+    """Time oracle.verify on whole-chain samples of one input set until ~seconds elapse."""
+    from oracle import verify as OV
+    m = OV.MODE_BLOCK if mode == "block" else OV.MODE_SAMPLE
+    Bn, L = inp["B"], inp["L"]
+    chains_done, t_total, calls = 0, 0.0, 0
+    per_call = Bn if max_chains is None else min(Bn, max_chains)
+    rng = np.random.Generator(np.random.PCG64(0))
+    while t_total < seconds:
+        ch = np.sort(rng.choice(Bn, per_call, replace=False))
+        t0 = time.perf_counter()
+        OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], seed + calls,
+                  m, chains=ch)
+        t_total += time.perf_counter() - t0
+        chains_done += per_call
+        calls += 1
+    return chains_done * L / t_total, chains_done, t_total
+
+
+def run_reference(args, world, rank):
+    """Reference arm: the CPU oracle as it stands, on the host cores, same workload/metric."""
+    if rank != 0:
+        return
+    cfg = W.VERIFY_CONFIGS[args.workload]
+    inp = W.make_verify_inputs(args.workload)
+    from oracle import verify as OV
+    m = OV.MODE_BLOCK if args.mode == "block" else OV.MODE_SAMPLE
+    # calibrate: chains per step so that warmup + steps take ~120 s at most
+    t0 = time.perf_counter()
+    OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], 0, m,
+              chains=np.arange(1))
+    t1 = time.perf_counter() - t0
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    per_step = int(max(1, min(cfg["B"], budget / max(t1, 1e-6))))
+    rng = np.random.Generator(np.random.PCG64(1))
+    for w in range(args.warmup):
+        OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], w, m,
+                  chains=rng.choice(cfg["B"], per_step, replace=False))
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], 1000 + s, m,
+                  chains=rng.choice(cfg["B"], per_step, replace=False))
+    dt = time.perf_counter() - t0
+    value = args.steps * per_step * cfg["L"] / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": "%s verify, %s mode" % (W.describe(args.workload), args.mode)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "%d chain(s) of the %s batch per step (oracle.verify, numpy fp64)"
+                                   % (per_step, args.workload)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+
+    import torch
+    import __graft_entry__ as G
+    G.build()
+    from paper_2606_13426_gb300 import api, binding
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    cfg = W.VERIFY_CONFIGS[args.workload]
+    Bn, L, d, dt_name = cfg["B"], cfg["L"], cfg["d"], cfg["dtype"]
+    tdt = torch.bfloat16 if dt_name == "bf16" else torch.float32
+    set_bytes = W.main_pass_bytes(Bn, L, d, dt_name)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size if hasattr(
+        torch.cuda.get_device_properties(dev), "L2_cache_size") else 129 * 2 ** 20
+    n_sets = max(1, min(N_SETS, math.ceil(4 * l2 / set_bytes))) if set_bytes < 4 * l2 else 1
+
+    def to_dev(inp, name):
+        if dt_name == "bf16":
+            return torch.from_numpy(inp[name + "_bits"].view(np.int16)).to(dev).view(torch.bfloat16)
+        return torch.from_numpy(inp[name]).to(dev)
+
+    sets = []
+    host0 = None
+    for i in range(n_sets):
+        inp = W.make_verify_inputs(args.workload, seed=cfg["seed"] + 100 * i + 7 * rank)
+        sets.append(dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"),
+                         mp=to_dev(inp, "mu_draft"), sigma=torch.from_numpy(inp["sigma"]).to(dev)))
+        if i == 0:
+            host0 = inp
+    outs = dict(accepted_len=torch.empty(Bn, dtype=torch.int32, device=dev),
+                y=torch.empty(Bn, d, dtype=tdt, device=dev),
+                status=torch.empty(Bn, dtype=torch.int32, device=dev))
+    ws = api.make_workspace(Bn, L, d, tdt, dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i):
+        s = sets[i % n_sets]
+        api.verify(s["x"], s["mq"], s["mp"], s["sigma"], seed=i, mode=args.mode,
+                   with_ratios=False, workspace=ws, out=outs)
+
+    G_STEPS = min(args.steps, 256)
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            step(i)
+    torch.cuda.synchronize()
+    binding.sdv_timing_enable(G_STEPS)
+
+    graphs = []
+    use_graph = not args.no_graph
+    if use_graph:
+        try:
+            reps, rem = divmod(args.steps, G_STEPS)
+            g_main = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_main, stream=stream):
+                for i in range(G_STEPS):
+                    step(i)
+            graphs = [g_main] * reps
+            if rem:
+                g_rem = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g_rem, stream=stream):
+                    for i in range(rem):
+                        step(i)
+                graphs.append(g_rem)
+            for g in graphs[:1]:
+                g.replay()
+            torch.cuda.synchronize()
+        except Exception as e:  # capture unsupported: time eager launches instead
+            sys.stderr.write("graph capture failed (%s); timing eager launches\n" % e)
+            use_graph = False
+            torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        if use_graph:
+            for g in graphs:
+                g.replay()
+        else:
+            for i in range(args.steps):
+                step(i)
+        ev1.record(stream)
+    torch.cuda.synchronize()
+    ms_total = ev0.elapsed_time(ev1)
+    clk = clocks.stop()
+    n_timed = G_STEPS if use_graph and args.steps % G_STEPS == 0 else min(args.steps, G_STEPS)
+    k1_ms, k2_ms, k4_ms = (v / n_timed for v in binding.sdv_timing_read(n_timed))
+    binding.sdv_timing_enable(0)
+    if pg:
+        t = torch.tensor([ms_total], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms_total = float(t.item())
+        pg.barrier()
+    ms_step = ms_total / args.steps
+    value = world * Bn * L / (ms_step * 1e-3)
+
+    # mean tau per target call, block and sample, over the input sets
+    taus = {}
+    for mode in ("block", "sample"):
+        acc = []
+        for i, s in enumerate(sets):
+            r = api.verify(s["x"], s["mq"], s["mp"], s["sigma"], seed=10_000 + i, mode=mode,
+                           with_ratios=False, workspace=ws)
+            acc.append(r["accepted_len"].cpu().numpy())
+        taus[mode] = float(np.concatenate(acc).mean() + 1.0)
+
+    # end to end: pinned host window in, accepted lengths and states out
+    sig_shape = tuple(host0["sigma"].shape)
+    hx = torch.empty(Bn, L, d, dtype=tdt, pin_memory=True)
+    hq = torch.empty_like(hx, pin_memory=True)
+    hp = torch.empty_like(hx, pin_memory=True)
+    if dt_name == "bf16":
+        for h, n in ((hx, "x_draft"), (hq, "mu_target"), (hp, "mu_draft")):
+            h.view(torch.int16).copy_(torch.from_numpy(host0[n + "_bits"].view(np.int16)))
+    else:
+        hx.copy_(torch.from_numpy(host0["x_draft"]))
+        hq.copy_(torch.from_numpy(host0["mu_target"]))
+        hp.copy_(torch.from_numpy(host0["mu_draft"]))
+    hs = torch.from_numpy(host0["sigma"]).pin_memory()
+    dbufs = api.make_device_buffers(Bn, L, d, tdt, sig_shape, device=dev)
+    e2e_steps = max(20, min(400, args.steps // 50))
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            api.verify_host(hx, hq, hp, hs, i, args.mode, dev_bufs=dbufs)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for i in range(e2e_steps):
+            api.verify_host(hx, hq, hp, hs, i, args.mode, dev_bufs=dbufs)
+        e2e_s = (time.perf_counter() - t0) / e2e_steps
+    h2d = 3 * hx.numel() * hx.element_size() + hs.numel() * 4
+    d2h = Bn * 4 + Bn * d * hx.element_size()
+
+    hbm_peak, peak_kind = peaks()
+    k1_bytes = set_bytes
+    achieved = k1_bytes / (k1_ms * 1e-3) / 1e9
+    kernel_src = os.path.join(ROOT, "paper_2606_13426_gb300", "csrc", "sdv_verify.cu")
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32" if dt_name == "f32" else "bf16",
+        "data": "synthetic",
+        "config": {"workload": "%s verify (B=%d, L=%d, d=%d %s), %s mode"
+                               % (args.workload, Bn, L, d, dt_name, args.mode),
+                   "global_batch": world * Bn, "window": L, "dim": d,
+                   "parallelism": "replicas" if world > 1 else "single-gpu",
+                   "l2": "%d rotating input sets, %.0f MB > L2 %.0f MB" % (
+                       n_sets, n_sets * set_bytes / 1e6, l2 / 1e6) if n_sets > 1 else
+                   "one input set of %.0f MB > L2" % (set_bytes / 1e6),
+                   "cuda_graph": use_graph},
+        "hbm_gbs_step": (set_bytes / (ms_step * 1e-3)) / 1e9,
+        "mean_tau_block": taus["block"], "mean_tau_sample": taus["sample"],
+        "phase_us": {"log_ratio_pass": 1e3 * k1_ms, "scan_usample": 1e3 * k2_ms,
+                     "residual": 1e3 * k4_ms},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                     "kernel": "k_ratio_partials (log-ratio pass)",
+                     "traffic": profile_traffic(kernel_src)},
+        "e2e": {"value": world * Bn * L / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        rate, nch, tsec = cpu_oracle_rate(host0, 0, args.mode, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
+                                "sample": "%d chains of the %s batch through oracle.verify "
+                                          "(numpy fp64, one thread), %.1f s"
+                                          % (nch, args.workload, tsec)}
+    if rank == 0:
+        print(json.dumps(line))
+    if pg:
+        pg.barrier()
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

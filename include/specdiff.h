@@ -1,0 +1,228 @@
+/*
+ * specdiff.h - C ABI of the GB300 (sm_103a) verification step of speculative
+ * diffusion sampling ("Accelerating Speculative Diffusions via Block
+ * Verification").
+ *
+ * One verification call takes, for B independent chains, a window of L drafted
+ * Gaussian transition steps in dimension d:
+ *   x_draft   [B, L, d]  yhat_{k+1} .. yhat_{k+L}   drafted states
+ *   mu_target [B, L, d]  m^q_{k}   .. m^q_{k+L-1}  target means  (Eq. target-distribution)
+ *   mu_draft  [B, L, d]  m^p_{k}   .. m^p_{k+L-1}  draft means   (Eq. draft-distribution)
+ *   sigma     [B, L]     sigma_{k} .. sigma_{k+L-1} shared std of both kernels
+ * and returns, per chain, the accepted length tau-1 and the state emitted at
+ * step k+tau (residual draw, bonus step or last accepted draft).
+ *
+ * Conventions for every entry point:
+ *   - Array pointers are DEVICE pointers owned by the caller unless stated
+ *     otherwise; nothing is retained after the call returns.  All arrays are
+ *     dense row-major (C order) with the shapes given.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     rejected call returns a negative SDV_E* code and launches nothing.
+ *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = the
+ *     legacy default stream).  No call synchronises, allocates device memory
+ *     or traps on the device.  A launch failure returns SDV_ECUDA;
+ *     sdv_last_cuda_error() then gives the cudaError_t.
+ *   - Results are a pure function of (inputs, seed, options): reductions use a
+ *     fixed order and no floating-point atomics.
+ *   - Random numbers come from Philox4x32-10 (Salmon et al., SC'11) keyed by
+ *     the 64-bit seed, with counter (chain b, index, stream id, sub):
+ *       coin eta_j of chain b, step j (0-based) : (b, j, 0, 0) word 0
+ *       residual uniform w of chain b          : (b, 0, 1, 0) word 0
+ *       residual Gaussian G, element i         : (b, i/4, 2, 0) words -> Box-Muller pairs
+ *       bonus-step Gaussian                    : (b, i/4, 3, 0)
+ *     uniform(x) = (x + 1/2) 2^-32;  Box-Muller on (w0,w1) and (w2,w3).
+ *   - Arithmetic is fp32 (bf16 inputs are widened exactly); outputs y_out use
+ *     the input dtype.
+ */
+#ifndef SPECDIFF_H
+#define SPECDIFF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- return codes ---------------------------------------------------- */
+#define SDV_OK            0
+#define SDV_EINVAL       (-1)  /* bad size, mode, dtype, option or NULL pointer */
+#define SDV_EALIGN       (-2)  /* a pointer is not aligned to its element size  */
+#define SDV_ECUDA        (-3)  /* a kernel launch failed (see sdv_last_cuda_error) */
+#define SDV_ENOWORKSPACE (-4)  /* workspace NULL or smaller than required       */
+
+/* ---- enums ----------------------------------------------------------- */
+#define SDV_MODE_SAMPLE 0      /* Algorithm token-verification (sample verification) */
+#define SDV_MODE_BLOCK  1      /* Algorithm block-verification                     */
+
+#define SDV_F32  0             /* float32 x / means / y_out */
+#define SDV_BF16 1             /* bfloat16 x / means / y_out (fp32 arithmetic) */
+
+#define SDV_RESIDUAL_DECOMPOSITION 0  /* Algorithm decomposition-res + u-sample */
+#define SDV_RESIDUAL_REFLECTION    1  /* Algorithm reflect-res (sample verification only) */
+
+/* per-chain status bits (status_out) */
+#define SDV_STATUS_ZERO_DELTA     1u  /* |Delta_tau| = 0 at the residual: y = m^q + sigma G      */
+#define SDV_STATUS_NONFINITE      2u  /* a log ratio, |Delta| or sigma in the window is not finite */
+#define SDV_STATUS_USAMPLE_RANGE  4u  /* U-sampler found no bracket (U clamped)                  */
+
+#define SDV_MAX_L 64           /* largest supported window */
+
+typedef void *sdv_stream_t;    /* cudaStream_t */
+
+/* Library identification and error text. */
+const char *sdv_version(void);
+const char *sdv_strerror(int code);
+/* cudaError_t of the last SDV_ECUDA returned on this host thread (0 if none). */
+int sdv_last_cuda_error(void);
+
+/*
+ * Bytes of device workspace sdv_verify / sdv_verify_ex / sdv_log_ratios need
+ * for (B, L, d, dtype); 0 for invalid sizes.  The caller allocates it (any
+ * 256-byte aligned device buffer) and may reuse it across calls on one stream.
+ */
+size_t sdv_workspace_bytes(int B, int L, int64_t d, int dtype);
+
+/*
+ * sdv_verify - the whole verification step (log ratios, acceptance rule,
+ * residual draw), Algorithms token-/block-verification, decomposition-res and
+ * u-sample, in the log form of App. "Density ratio calculations":
+ *   Delta_j = (m^p - m^q)/sigma, Z_j = (yhat - m^p)/sigma,
+ *   ell_j = log N(Z+Delta)/N(Z) = -Z^T Delta - |Delta|^2/2.
+ * sample: tau = first j with eta_j >= min{1, e^ell_j}, else L+1.
+ * block:  log alpha_j = min{0, log alpha_{j-1} + ell_j};
+ *         h_j = v_j/(v_j + 1 - alpha_j) (j < L), h_L = alpha_L,
+ *         v_j = alpha_j Phi(log alpha_j/D_{j+1} + D_{j+1}/2) - Phi(log alpha_j/D_{j+1} - D_{j+1}/2);
+ *         tau = 1 + max{j : eta_j < h_j}, the max being 0 when no coin succeeds.
+ * residual (tau <= L): y = m^q_tau + sigma_tau (U e + G - e e^T G),
+ *         e = Delta_tau/|Delta_tau|, U = Psi_alpha^{-1}(w), alpha = alpha_{tau-1}
+ *         (1 in sample mode), Psi_alpha of Eq. u-cdf.
+ * full accept (tau = L+1): y = x_draft[b, L-1].
+ *
+ *   x_draft, mu_target, mu_draft : [B, L, d] of `dtype`
+ *   sigma          : fp32, element (b, j) at sigma[b*sigma_stride_b + j];
+ *                    sigma_stride_b = 0 shares one row [L] across chains
+ *   B >= 1, 1 <= L <= SDV_MAX_L, d >= 1
+ *   seed           : Philox key; mode: SDV_MODE_*
+ *   accepted_len   : [B] int32 out, tau - 1 in [0, L]
+ *   y_out          : [B, d] out, `dtype`
+ *   log_ratio_out  : [B, L] fp32 out or NULL: ell_j (0 past the window)
+ *   delta_norm_out : [B, L] fp32 out or NULL: |Delta_j|
+ *   status_out     : [B] uint32 out or NULL: SDV_STATUS_* bits
+ *   workspace      : >= sdv_workspace_bytes(B, L, d, dtype) bytes of device memory
+ * Inputs must not alias outputs.
+ */
+int sdv_verify(const void *x_draft, const void *mu_target, const void *mu_draft,
+               const float *sigma, int64_t sigma_stride_b,
+               int B, int L, int64_t d, int dtype,
+               uint64_t seed, int mode,
+               int32_t *accepted_len, void *y_out,
+               float *log_ratio_out, float *delta_norm_out, uint32_t *status_out,
+               void *workspace, size_t workspace_bytes, sdv_stream_t stream);
+
+/*
+ * sdv_verify_ex - sdv_verify plus the options the end-to-end sampler needs
+ * (Algorithm full-block-verification):
+ *   L_eff          : [B] int32 or NULL: window length gamma_k of each chain,
+ *                    0 <= L_eff[b] <= L; steps j >= L_eff[b] are never read.
+ *                    0 marks an inactive chain: accepted_len = 0, its y_out row
+ *                    and status are not written.
+ *   mu_target_bonus: [B, d] `dtype` or NULL: m^q_{k+gamma_k}; when given, a
+ *                    full accept emits the bonus step y = m^q_bonus + sigma_bonus G_bonus
+ *   sigma_bonus    : [B] fp32 (required with mu_target_bonus)
+ *   residual_kind  : SDV_RESIDUAL_DECOMPOSITION or SDV_RESIDUAL_REFLECTION
+ *                    (reflection needs mode == SDV_MODE_SAMPLE)
+ *   omega          : temperature (App. Temperature): the acceptance rule uses
+ *                    ell/omega^2, block h_j and alpha_res take the tempered
+ *                    alpha; omega = 1 is the exact method
+ *   chain_aux_out  : [B, 4] fp32 out or NULL: (U, log alpha_res, |Delta_tau|,
+ *                    sigma_tau); NaN where not applicable
+ */
+int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_draft,
+                  const float *sigma, int64_t sigma_stride_b,
+                  int B, int L, int64_t d, int dtype,
+                  uint64_t seed, int mode,
+                  const int32_t *L_eff,
+                  const void *mu_target_bonus, const float *sigma_bonus,
+                  int residual_kind, float omega,
+                  int32_t *accepted_len, void *y_out,
+                  float *log_ratio_out, float *delta_norm_out, uint32_t *status_out,
+                  float *chain_aux_out,
+                  void *workspace, size_t workspace_bytes, sdv_stream_t stream);
+
+/*
+ * sdv_log_ratios - only the fused reduction over d (App. "Density ratio
+ * calculations"): ell_j = -Z_j^T Delta_j - |Delta_j|^2/2 and |Delta_j| for
+ * every (b, j) with j < L_eff[b] (all j if L_eff is NULL; 0 elsewhere).
+ * Shapes and dtype as in sdv_verify; log_ratio_out and delta_norm_out are
+ * [B, L] fp32 and required.
+ */
+int sdv_log_ratios(const void *x_draft, const void *mu_target, const void *mu_draft,
+                   const float *sigma, int64_t sigma_stride_b,
+                   int B, int L, int64_t d, int dtype, const int32_t *L_eff,
+                   float *log_ratio_out, float *delta_norm_out,
+                   void *workspace, size_t workspace_bytes, sdv_stream_t stream);
+
+/*
+ * sdv_accept_scan - only the acceptance rule over the window
+ * (Algorithms token-/block-verification and their temperature variants),
+ * from given log ratios and norms:
+ *   log_ratio, delta_norm : [B, L] fp32 (ell_j, |Delta_j|); L_eff as above
+ *   tau_out               : [B] int32 out, tau in [1, L_eff+1] (0 if inactive)
+ *   log_alpha_res_out     : [B] fp32 out or NULL, log alpha_{tau-1} (0 in sample mode)
+ * Coins eta_j are drawn from `seed` exactly as in sdv_verify.
+ */
+int sdv_accept_scan(const float *log_ratio, const float *delta_norm,
+                    int B, int L, const int32_t *L_eff, uint64_t seed, int mode, float omega,
+                    int32_t *tau_out, float *log_alpha_res_out, sdv_stream_t stream);
+
+/*
+ * sdv_usample - only the residual's 1-D draw, U = Psi_alpha^{-1}(w)
+ * (Proposition decomposition, Eq. u-cdf, Algorithm u-sample), for n
+ * independent items:
+ *   delta_norm [n] fp32 (> 0), log_alpha [n] fp32 (<= 0),
+ *   w_bits [n] uint32: the 32-bit Philox word, w = (w_bits + 1/2) 2^-32,
+ *   U_out [n] fp32 out, status_out [n] uint32 out or NULL.
+ */
+int sdv_usample(const float *delta_norm, const float *log_alpha, const uint32_t *w_bits,
+                int n, float *U_out, uint32_t *status_out, sdv_stream_t stream);
+
+/*
+ * sdv_philox - raw Philox4x32-10 blocks: out[i][0..3] for counter ctr[i][0..3]
+ * and key (seed lo, seed hi); ctr and out are [n][4] uint32 device arrays.
+ */
+int sdv_philox(const uint32_t *ctr, uint64_t seed, int n, uint32_t *out, sdv_stream_t stream);
+
+/*
+ * sdv_normals - the Gaussian noise the kernels draw: out[b][i] for chain b,
+ * element i on Philox stream `stream_id` and sub-counter `sub`
+ * (counter (b, i/4, stream_id, sub), Box-Muller), fp32 [B, d] out.
+ */
+int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub,
+                float *out, sdv_stream_t stream);
+
+/*
+ * Profiling aid (not part of the method): when enabled, every later
+ * sdv_verify / sdv_verify_ex call made on this host thread records four CUDA
+ * events on its stream - before the log-ratio pass, after it, after the
+ * acceptance scan, after the residual write - into a ring of `slots` entries.
+ * The records are ordinary stream work, so they are captured into a CUDA graph
+ * like the kernels.  The events are created here (host objects; no device
+ * memory).  slots = 0 disables timing and destroys the events.
+ */
+int sdv_timing_enable(int slots);
+
+/*
+ * Waits for the events of the last `n_calls` recorded calls (1 <= n_calls <=
+ * slots) and writes their summed phase times in milliseconds:
+ * ms3[0] log-ratio pass (K1), ms3[1] acceptance scan + U-sampler (K2),
+ * ms3[2] residual dot + write (K4).  SDV_EINVAL if timing is off or fewer
+ * calls were recorded.
+ */
+int sdv_timing_read(int n_calls, float *ms3);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPECDIFF_H */

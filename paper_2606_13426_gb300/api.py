@@ -1,0 +1,185 @@
+"""Torch-facing helpers over the C ABI: allocate outputs and workspace, pass pointers.
+
+PyTorch provides device memory and the current stream only; every step of the
+verification path runs in libspecdiff's kernels.  Inputs must be CUDA tensors
+(this module never computes anything itself and has no CPU path).
+"""
+import torch
+
+from . import binding as B
+
+_DTYPES = {torch.float32: B.SDV_F32, torch.bfloat16: B.SDV_BF16}
+_MODES = {"sample": B.SDV_MODE_SAMPLE, "block": B.SDV_MODE_BLOCK,
+          B.SDV_MODE_SAMPLE: B.SDV_MODE_SAMPLE, B.SDV_MODE_BLOCK: B.SDV_MODE_BLOCK}
+_RESIDUALS = {"decomposition": B.SDV_RESIDUAL_DECOMPOSITION,
+              "reflection": B.SDV_RESIDUAL_REFLECTION}
+
+
+def _ptr(t):
+    return 0 if t is None else t.data_ptr()
+
+
+def _stream():
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None and (not t.is_cuda or not t.is_contiguous()):
+            raise ValueError("libspecdiff needs contiguous CUDA tensors")
+
+
+def workspace_bytes(B_, L, d, dtype=torch.float32):
+    return B.sdv_workspace_bytes(B_, L, d, _DTYPES[dtype])
+
+
+def make_workspace(B_, L, d, dtype=torch.float32, device="cuda"):
+    return torch.empty(max(workspace_bytes(B_, L, d, dtype), 256), dtype=torch.uint8, device=device)
+
+
+def _sigma_args(sigma, Bn, L):
+    if sigma.dim() == 1:
+        if sigma.shape[0] != L:
+            raise ValueError("sigma [L] expected")
+        return sigma, 0
+    if tuple(sigma.shape) != (Bn, L):
+        raise ValueError("sigma [B, L] expected")
+    return sigma, L
+
+
+def verify(x_draft, mu_target, mu_draft, sigma, seed, mode="block", *, L_eff=None,
+           mu_target_bonus=None, sigma_bonus=None, residual="decomposition", omega=1.0,
+           with_ratios=True, with_aux=False, workspace=None, out=None):
+    """One verification call (sdv_verify_ex) on [B, L, d] CUDA tensors; returns a dict of outputs."""
+    _need_cuda(x_draft, mu_target, mu_draft, sigma, L_eff, mu_target_bonus, sigma_bonus)
+    Bn, L, d = x_draft.shape
+    dt = x_draft.dtype
+    if mu_target.dtype != dt or mu_draft.dtype != dt or dt not in _DTYPES:
+        raise ValueError("x_draft, mu_target, mu_draft must share a float32/bfloat16 dtype")
+    if sigma.dtype != torch.float32:
+        raise ValueError("sigma must be float32")
+    sigma, sstride = _sigma_args(sigma, Bn, L)
+    dev = x_draft.device
+    if out is None:
+        out = {}
+    acc = out.get("accepted_len")
+    if acc is None:
+        acc = torch.empty(Bn, dtype=torch.int32, device=dev)
+    y = out.get("y")
+    if y is None:
+        y = torch.empty(Bn, d, dtype=dt, device=dev)
+    lr = dn = None
+    if with_ratios:
+        lr = out.get("log_ratio")
+        lr = torch.empty(Bn, L, dtype=torch.float32, device=dev) if lr is None else lr
+        dn = out.get("delta_norm")
+        dn = torch.empty(Bn, L, dtype=torch.float32, device=dev) if dn is None else dn
+    st = out.get("status")
+    st = torch.empty(Bn, dtype=torch.int32, device=dev) if st is None else st
+    aux = None
+    if with_aux:
+        aux = out.get("aux")
+        aux = torch.empty(Bn, 4, dtype=torch.float32, device=dev) if aux is None else aux
+    if workspace is None:
+        workspace = make_workspace(Bn, L, d, dt, dev)
+    B.sdv_verify_ex(_ptr(x_draft), _ptr(mu_target), _ptr(mu_draft), _ptr(sigma), sstride,
+                    Bn, L, d, _DTYPES[dt], int(seed) & 0xFFFFFFFFFFFFFFFF, _MODES[mode],
+                    _ptr(L_eff), _ptr(mu_target_bonus), _ptr(sigma_bonus),
+                    _RESIDUALS[residual], float(omega),
+                    _ptr(acc), _ptr(y), _ptr(lr), _ptr(dn), _ptr(st), _ptr(aux),
+                    _ptr(workspace), workspace.numel(), _stream())
+    res = dict(accepted_len=acc, y=y, status=st)
+    if with_ratios:
+        res.update(log_ratio=lr, delta_norm=dn)
+    if with_aux:
+        res["aux"] = aux
+    return res
+
+
+def verify_host(x_draft, mu_target, mu_draft, sigma, seed, mode="block", *, dev_bufs=None):
+    """End-to-end call from pinned host tensors: copy in, verify, copy accepted_len and y back.
+
+    ``dev_bufs`` (from ``make_device_buffers``) holds the device copies and
+    outputs so repeated calls allocate nothing.  Returns (accepted_len, y) as
+    host tensors, synchronised.
+    """
+    Bn, L, d = x_draft.shape
+    if dev_bufs is None:
+        dev_bufs = make_device_buffers(Bn, L, d, x_draft.dtype, sigma.shape)
+    db = dev_bufs
+    db["x"].copy_(x_draft, non_blocking=True)
+    db["mq"].copy_(mu_target, non_blocking=True)
+    db["mp"].copy_(mu_draft, non_blocking=True)
+    db["sigma"].copy_(sigma, non_blocking=True)
+    verify(db["x"], db["mq"], db["mp"], db["sigma"], seed, mode, with_ratios=False,
+           workspace=db["ws"], out=db)
+    db["h_acc"].copy_(db["accepted_len"], non_blocking=True)
+    db["h_y"].copy_(db["y"], non_blocking=True)
+    torch.cuda.current_stream().synchronize()
+    return db["h_acc"], db["h_y"]
+
+
+def make_device_buffers(Bn, L, d, dtype, sigma_shape, device="cuda"):
+    return dict(
+        x=torch.empty(Bn, L, d, dtype=dtype, device=device),
+        mq=torch.empty(Bn, L, d, dtype=dtype, device=device),
+        mp=torch.empty(Bn, L, d, dtype=dtype, device=device),
+        sigma=torch.empty(*sigma_shape, dtype=torch.float32, device=device),
+        accepted_len=torch.empty(Bn, dtype=torch.int32, device=device),
+        y=torch.empty(Bn, d, dtype=dtype, device=device),
+        status=torch.empty(Bn, dtype=torch.int32, device=device),
+        ws=make_workspace(Bn, L, d, dtype, device),
+        h_acc=torch.empty(Bn, dtype=torch.int32, pin_memory=True),
+        h_y=torch.empty(Bn, d, dtype=dtype, pin_memory=True),
+    )
+
+
+def log_ratios(x_draft, mu_target, mu_draft, sigma, L_eff=None, workspace=None):
+    """ell_j and |Delta_j| only (sdv_log_ratios)."""
+    _need_cuda(x_draft, mu_target, mu_draft, sigma, L_eff)
+    Bn, L, d = x_draft.shape
+    sigma, sstride = _sigma_args(sigma, Bn, L)
+    lr = torch.empty(Bn, L, dtype=torch.float32, device=x_draft.device)
+    dn = torch.empty_like(lr)
+    if workspace is None:
+        workspace = make_workspace(Bn, L, d, x_draft.dtype, x_draft.device)
+    B.sdv_log_ratios(_ptr(x_draft), _ptr(mu_target), _ptr(mu_draft), _ptr(sigma), sstride,
+                     Bn, L, d, _DTYPES[x_draft.dtype], _ptr(L_eff), _ptr(lr), _ptr(dn),
+                     _ptr(workspace), workspace.numel(), _stream())
+    return lr, dn
+
+
+def accept_scan(log_ratio, delta_norm, seed, mode="block", L_eff=None, omega=1.0):
+    """tau and log alpha_{tau-1} from given ell, |Delta| (sdv_accept_scan)."""
+    _need_cuda(log_ratio, delta_norm, L_eff)
+    Bn, L = log_ratio.shape
+    tau = torch.empty(Bn, dtype=torch.int32, device=log_ratio.device)
+    la = torch.empty(Bn, dtype=torch.float32, device=log_ratio.device)
+    B.sdv_accept_scan(_ptr(log_ratio), _ptr(delta_norm), Bn, L, _ptr(L_eff),
+                      int(seed) & 0xFFFFFFFFFFFFFFFF, _MODES[mode], float(omega),
+                      _ptr(tau), _ptr(la), _stream())
+    return tau, la
+
+
+def usample(delta_norm, log_alpha, w_bits):
+    """U = Psi_alpha^{-1}(w) for each item (sdv_usample); w_bits is int32 holding uint32 words."""
+    _need_cuda(delta_norm, log_alpha, w_bits)
+    n = delta_norm.numel()
+    U = torch.empty(n, dtype=torch.float32, device=delta_norm.device)
+    st = torch.empty(n, dtype=torch.int32, device=delta_norm.device)
+    B.sdv_usample(_ptr(delta_norm), _ptr(log_alpha), _ptr(w_bits), n, _ptr(U), _ptr(st), _stream())
+    return U, st
+
+
+def philox(ctr, seed):
+    """Raw Philox4x32-10 blocks for counters ctr [n, 4] (int32 holding uint32 words)."""
+    _need_cuda(ctr)
+    out = torch.empty_like(ctr)
+    B.sdv_philox(_ptr(ctr), int(seed) & 0xFFFFFFFFFFFFFFFF, ctr.shape[0], _ptr(out), _stream())
+    return out
+
+
+def normals(seed, Bn, d, stream_id, sub=0, device="cuda"):
+    out = torch.empty(Bn, d, dtype=torch.float32, device=device)
+    B.sdv_normals(int(seed) & 0xFFFFFFFFFFFFFFFF, Bn, d, stream_id, sub, _ptr(out), _stream())
+    return out

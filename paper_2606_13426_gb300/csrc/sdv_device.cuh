@@ -1,0 +1,290 @@
+// sdv_device.cuh - device-side building blocks of the verification step (sm_103a).
+//
+//  * Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) and the uniform /
+//    Box-Muller transforms of the counter layout documented in specdiff.h.
+//  * log Phi and the scaled log-CDF g(a) = log Phi(a) + a^2/2, its derivative
+//    g'(s) = lambda(s) + s (lambda = phi/Phi, the inverse Mills ratio), and
+//    differences g(hi) - g(hi - h) by 8-point Gauss-Legendre quadrature.
+//  * The block-verification acceptance probability h_j (Algorithm
+//    block-verification) in log form (App. "Density ratio calculations").
+//  * The residual's 1-D draw U = Psi_alpha^{-1}(w) (Prop. decomposition,
+//    Eq. u-cdf, Algorithm u-sample) as a warp-cooperative multisection.
+//
+// Everything is fp32: GB300's fp64 rate is a small fraction of its fp32 rate.
+// The forms below avoid the cancellations that fp32 would otherwise suffer:
+//  - v = alpha Phi(a+) - Phi(a-) is written as alpha Phi(a+) (1 - e^{x0}) with
+//    x0 = log(Phi(a-)/(alpha Phi(a+))) = g(a-) - g(a+), exact because
+//    log alpha + a-^2/2 = a+^2/2 (a+- = log alpha / D +- D/2);
+//  - Psi near its upper end a+ (where its density vanishes) is evaluated as a
+//    complement, 1 - Psi(a+ - t) = int_0^t phi(a- - s) expm1(D s) ds / v,
+//    which has a positive integrand (alpha phi(u) - phi(u - D) =
+//    phi(u - D) expm1(D (a+ - u)));
+//  - for s < -4, lambda(s) + s = 1/(x + 2/(x + 3/(x + ...))), x = -s, which is
+//    Laplace's continued fraction for the Mills ratio with its first term
+//    cancelled analytically.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+namespace sdv {
+
+// ---------------------------------------------------------------- Philox
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
+
+enum : uint32_t {
+  kStreamCoin = 0,
+  kStreamUSample = 1,
+  kStreamResid = 2,
+  kStreamBonus = 3,
+  kStreamDraft = 4,
+  kStreamInit = 5,
+  kStreamEM = 6,
+};
+
+// Ten rounds of the Philox4x32 S-box: (c0,c1,c2,c3) -> (hi(M1 c2)^c1^k0,
+// lo(M1 c2), hi(M0 c0)^c3^k1, lo(M0 c0)); the key is bumped by the Weyl
+// constants between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += kPhiloxW0;
+      k1 += kPhiloxW1;
+    }
+    const uint32_t lo0 = kPhiloxM0 * c.x;
+    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x);
+    const uint32_t lo1 = kPhiloxM1 * c.z;
+    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+  }
+  return c;
+}
+
+__device__ __forceinline__ uint4 philox_block(uint64_t seed, uint32_t c0, uint32_t c1,
+                                              uint32_t c2, uint32_t c3) {
+  return philox4x32_10(make_uint4(c0, c1, c2, c3), (uint32_t)seed, (uint32_t)(seed >> 32));
+}
+
+// log u for u = (x + 1/2) 2^-32; the upper half goes through 1 - u, which is
+// exact in the integer domain, so log u keeps full relative accuracy near 1.
+__device__ __forceinline__ float log_uniform(uint32_t x) {
+  if (x < 0x80000000u) return logf(((float)x + 0.5f) * 0x1p-32f);
+  return log1pf(-(((float)(0xFFFFFFFFu - x) + 0.5f) * 0x1p-32f));
+}
+
+// Box-Muller on two words: (r cos 2 pi u1, r sin 2 pi u1), r = sqrt(-2 ln u0).
+__device__ __forceinline__ float2 box_muller(uint32_t w0, uint32_t w1) {
+  const float r = sqrtf(-2.0f * log_uniform(w0));
+  float s, c;
+  sincospif(((float)w1 + 0.5f) * 0x1p-31f, &s, &c);
+  return make_float2(r * c, r * s);
+}
+
+// Four normals of Philox block (b, blk, stream, sub): elements 4 blk .. 4 blk + 3.
+__device__ __forceinline__ float4 normals4(uint64_t seed, uint32_t b, uint32_t blk,
+                                           uint32_t stream, uint32_t sub) {
+  const uint4 w = philox_block(seed, b, blk, stream, sub);
+  const float2 z01 = box_muller(w.x, w.y);
+  const float2 z23 = box_muller(w.z, w.w);
+  return make_float4(z01.x, z01.y, z23.x, z23.y);
+}
+
+// ---------------------------------------------------------------- normal CDF helpers
+constexpr float kSqrtHalf = 0.70710678118654752f;
+constexpr float kHalfLog2Pi = 0.91893853320467274f;  // log(2 pi) / 2
+constexpr float kLn2 = 0.69314718055994531f;
+
+// 8-point Gauss-Legendre nodes / weights on [-1, 1] (positive half).
+static __constant__ float kGLx[4] = {0.18343464249564978f, 0.52553240991632899f,
+                                          0.79666647741362673f, 0.96028985649753618f};
+static __constant__ float kGLw[4] = {0.36268378337836166f, 0.31370664587788688f,
+                                          0.22238103445337443f, 0.10122853629037706f};
+
+// log Phi(a).
+__device__ __forceinline__ float log_ndtr(float a) {
+  if (a < -1.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf)) - 0.5f * a * a;
+  if (a > 0.0f) return log1pf(-0.5f * erfcf(a * kSqrtHalf));
+  return logf(0.5f * erfcf(-a * kSqrtHalf));
+}
+
+// g(a) = log Phi(a) + a^2/2 (moderate for a <= 0).
+__device__ __forceinline__ float gfun(float a) {
+  if (a < -1.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf));
+  return log_ndtr(a) + 0.5f * a * a;
+}
+
+// g'(s) = lambda(s) + s > 0.
+__device__ __forceinline__ float gprime(float s) {
+  if (s < -4.0f) {
+    const float x = -s;
+    float acc = x;
+#pragma unroll
+    for (int n = 16; n >= 2; --n) acc = x + (float)n / acc;
+    return 1.0f / acc;
+  }
+  return expf(-0.5f * s * s - kHalfLog2Pi - log_ndtr(s)) + s;
+}
+
+// g(hi) - g(hi - h) for h >= 0; the interval length is exactly h.
+__device__ __forceinline__ float gdiff(float hi, float h) {
+  if (h <= fmaxf(2.0f, 0.5f * fabsf(hi))) {
+    const float r = 0.5f * h, m = hi - r;
+    float acc = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      acc += kGLw[i] * (gprime(m + r * kGLx[i]) + gprime(m - r * kGLx[i]));
+    return r * acc;
+  }
+  const float lo = hi - h;
+  if (hi <= 0.0f) return gfun(hi) - gfun(lo);
+  return (log_ndtr(hi) - log_ndtr(lo)) + h * (hi - 0.5f * h);
+}
+
+// log(1 - e^x), x <= 0.
+__device__ __forceinline__ float log1mexp(float x) {
+  x = fminf(x, 0.0f);
+  return (x > -kLn2) ? logf(-expm1f(x)) : log1pf(-expf(x));
+}
+
+// log(e^y - 1), y >= 0.
+__device__ __forceinline__ float logexpm1(float y) {
+  return (y > 15.0f) ? y + log1pf(-expf(-y)) : logf(expm1f(y));
+}
+
+__device__ __forceinline__ float logaddexp(float a, float b) {
+  const float m = fmaxf(a, b);
+  if (m == -INFINITY) return -INFINITY;
+  return m + log1pf(expf(-fabsf(a - b)));
+}
+
+// log(Phi(b) - Phi(a)) for a < b.
+__device__ __forceinline__ float log_ndtr_interval(float a, float b) {
+  if (b <= 0.0f) return log_ndtr(b) + log1mexp(log_ndtr(a) - log_ndtr(b));
+  if (a >= 0.0f) return log_ndtr(-a) + log1mexp(log_ndtr(-b) - log_ndtr(-a));
+  return log1pf(-(expf(log_ndtr(a)) + expf(log_ndtr(-b))));
+}
+
+// ---------------------------------------------------------------- block verification
+// log h_j, h_j = v_j / (v_j + 1 - alpha_j), from log alpha_j (<= 0) and |Delta_{j+1}|.
+// Limits: alpha_j = 1 -> h = 1; alpha_j = 0 or |Delta_{j+1}| = 0 (alpha_j < 1) -> h = 0.
+__device__ __forceinline__ float block_log_h(float la, float Dn) {
+  if (isnan(la) || isnan(Dn)) return -INFINITY;
+  if (!(la < 0.0f)) return 0.0f;
+  if (la == -INFINITY || !(Dn > 0.0f)) return -INFINITY;
+  const float ap = la / Dn + 0.5f * Dn;
+  const float x0 = -gdiff(ap, Dn);              // log(Phi(a-) / (alpha Phi(a+)))
+  const float lv = la + log_ndtr(ap) + log1mexp(x0);
+  const float l1ma = log1mexp(la);              // log(1 - alpha)
+  return lv - logaddexp(lv, l1ma);
+}
+
+// ---------------------------------------------------------------- residual U-sampler
+struct UParams {
+  float D, la, ap, am;
+  float lv;   // log v
+  float lvn;  // log v - log phi(a-)
+};
+
+__device__ __forceinline__ UParams usample_setup(float D, float la) {
+  UParams P;
+  P.D = D;
+  P.la = la;
+  P.ap = la / D + 0.5f * D;
+  P.am = P.ap - D;
+  const float x0 = -gdiff(P.ap, D);
+  P.lv = la + log_ndtr(P.ap) + log1mexp(x0);
+  P.lvn = gfun(P.am) + kHalfLog2Pi + logexpm1(-x0);
+  return P;
+}
+
+// log Psi(a+ - t), t > 0.
+__device__ __forceinline__ float usample_log_psi(float t, const UParams& P) {
+  const float u = P.ap - t;
+  const float x = -gdiff(u, P.D) - P.D * t;     // log(Phi(u - D) / (alpha Phi(u)))
+  if (u < 0.0f)
+    return gfun(u) + log1mexp(x) - P.lvn + kHalfLog2Pi + 0.5f * t * (P.ap + u);
+  return P.la + log_ndtr(u) + log1mexp(x) - P.lv;
+}
+
+// log(1 - Psi(a+ - t)), t > 0.
+__device__ __forceinline__ float usample_log_1mpsi(float t, const UParams& P) {
+  if (P.D * t <= 1.0f && -P.am * t <= 4.0f) {
+    const float r = 0.5f * t;
+    float acc = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float s1 = r * (1.0f + kGLx[i]), s2 = r * (1.0f - kGLx[i]);
+      acc += kGLw[i] * (expf(P.am * s1 - 0.5f * s1 * s1) * expm1f(P.D * s1) +
+                        expf(P.am * s2 - 0.5f * s2 * s2) * expm1f(P.D * s2));
+    }
+    return logf(r * acc) - P.lvn;
+  }
+  const float u = P.ap - t;
+  const float lA = P.la + log_ndtr_interval(u, P.ap);
+  const float lB = log_ndtr_interval(u - P.D, P.am);
+  return lA + log1mexp(lB - lA) - P.lv;
+}
+
+// U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32.  Must be called by all 32
+// lanes of a warp with the same arguments; every lane returns U.
+// In t = a+ - u (Psi decreasing in t): a parallel doubling search over
+// t = 2^-12 .. 2^19 (the paper's bracket growth, all steps at once), then
+// five rounds of 32-way multisection (width / 2^25).  Lower half of w
+// compares log Psi with log w, upper half log(1 - Psi) with log(1 - w).
+__device__ __forceinline__ float usample_warp(float D, float la, uint32_t wbits,
+                                              uint32_t* status) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const UParams P = usample_setup(D, la);
+  const bool upper = wbits >= 0x80000000u;
+  const float target = upper ? logf(((float)(0xFFFFFFFFu - wbits) + 0.5f) * 0x1p-32f)
+                             : logf(((float)wbits + 0.5f) * 0x1p-32f);
+  auto below_w = [&](float t) -> bool {  // Psi(a+ - t) <= w
+    if (upper) return usample_log_1mpsi(t, P) >= target;
+    return usample_log_psi(t, P) <= target;
+  };
+  float tk = ldexpf(1.0f, lane - 12);
+  unsigned m = __ballot_sync(FULL, below_w(tk));
+  if (m == 0u) {
+    *status |= 4u;  // SDV_STATUS_USAMPLE_RANGE
+    return P.ap - ldexpf(1.0f, 19);
+  }
+  int f = __ffs(m) - 1;
+  float hi = __shfl_sync(FULL, tk, f);
+  float lo = (f == 0) ? 0.0f : __shfl_sync(FULL, tk, f - 1 < 0 ? 0 : f - 1);
+#pragma unroll 1
+  for (int round = 0; round < 5; ++round) {
+    const float h = (hi - lo) * (1.0f / 32.0f);
+    const float t = (lane < 31) ? lo + (float)(lane + 1) * h : hi;
+    const bool c = (lane < 31) ? below_w(t) : true;
+    m = __ballot_sync(FULL, c);
+    f = __ffs(m) - 1;
+    const float nhi = __shfl_sync(FULL, t, f);
+    const float nlo = __shfl_sync(FULL, t, f > 0 ? f - 1 : 0);
+    lo = (f == 0) ? lo : nlo;
+    hi = nhi;
+  }
+  return P.ap - 0.5f * (lo + hi);
+}
+
+// ---------------------------------------------------------------- element access
+template <typename T> struct Elem;
+template <> struct Elem<float> {
+  static __device__ __forceinline__ float load(const float* p) { return __ldg(p); }
+  static __device__ __forceinline__ void store(float* p, float v) { *p = v; }
+};
+template <> struct Elem<__nv_bfloat16> {
+  static __device__ __forceinline__ float load(const __nv_bfloat16* p) {
+    return __bfloat162float(__ldg(p));
+  }
+  static __device__ __forceinline__ void store(__nv_bfloat16* p, float v) {
+    *p = __float2bfloat16_rn(v);
+  }
+};
+
+}  // namespace sdv

@@ -1,0 +1,78 @@
+// sdv_host.h - internal launch parameters and workspace layout of libspecdiff.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/specdiff.h"
+
+namespace sdv {
+
+// K1: threads per CTA and 16-byte vectors per thread per tensor per sweep.
+constexpr int kK1Threads = 256;
+constexpr int kK1Vpt = 4;
+// K2: one warp per chain.
+constexpr int kK2Threads = 128;
+// K4: threads per CTA and elements of the rejected row per CTA.
+constexpr int kK4Threads = 256;
+constexpr int kK4Chunk = 4096;
+
+enum : int32_t {
+  kKindInactive = 0,
+  kKindResid = 1,      // decomposition residual
+  kKindReflect = 2,    // reflection residual
+  kKindZeroDelta = 3,  // |Delta_tau| = 0: m^q + sigma G
+  kKindCopy = 4,       // full accept, last draft row
+  kKindBonus = 5,      // full accept, bonus step
+};
+
+// Per-chain result of K2, consumed by K4 (32 bytes).
+struct ChainState {
+  int32_t tau;      // 1-based
+  int32_t row;      // row of the window K4 reads (tau-1, or the last draft)
+  float U;          // residual 1-D draw
+  float la_res;     // log alpha_{tau-1}
+  float sigma;      // sigma_tau
+  float inv_norm;   // 1/|delta_tau|, delta = m^p - m^q
+  float refl;       // 1 + 2 S1/S2 (reflection: y = x - delta * refl)
+  uint32_t status;
+  int32_t kind;
+  int32_t pad;
+};
+
+struct ScanArgs {
+  const float2* part;
+  int C;
+  const float* sigma;
+  int64_t sstride;
+  const float* ell_in;
+  const float* dn_in;
+  int B, L;
+  const int32_t* L_eff;
+  uint64_t seed;
+  int mode;
+  float inv_omega2;
+  int residual_kind;
+  bool has_bonus;
+  bool ratios_only;
+  float* ell_out;
+  float* dn_out;
+  int32_t* accepted_len;
+  int32_t* tau_out;
+  float* la_res_out;
+  uint32_t* status_out;
+  float* aux_out;
+  ChainState* state;
+};
+
+struct WsLayout {
+  int vpt1;        // K1 16-byte vectors per thread per tensor
+  int64_t chunk1;  // elements of a row per K1 tile
+  int C1;          // K1 tiles per row
+  int C4;          // K4 tiles per chain
+  size_t part_off, state_off, part4_off, total;
+};
+
+WsLayout ws_layout(int B, int L, int64_t d, int dtype);
+
+}  // namespace sdv

@@ -1,0 +1,830 @@
+// sdv_verify.cu - verification step of speculative diffusion sampling on sm_103a.
+//
+// Kernels of one sdv_verify call (all launched on the caller's stream):
+//   K1 ratio_partials : streams x, m^q, m^p once (16-byte loads) and reduces, per
+//                       (chain, step, d-chunk), S1 = sum (x - m^p)(m^p - m^q) and
+//                       S2 = sum (m^p - m^q)^2 (App. "Density ratio calculations":
+//                       Z^T Delta = S1/sigma^2, |Delta|^2 = S2/sigma^2).
+//   K2 scan           : one warp per chain: ell_j, |Delta_j|, the coins, sample or
+//                       block acceptance (Algorithms token-/block-verification), and
+//                       the residual draw U (Algorithm u-sample, warp multisection).
+//   K4a resid_dot     : sum_i delta_i G_i over the rejected row (e^T G up to 1/|delta|).
+//   K4b resid_write   : y = m^q + sigma (U e + G - e e^T G) (Algorithm decomposition-res),
+//                       or the reflection (Algorithm reflect-res), the bonus step,
+//                       or the last accepted draft.
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <algorithm>
+#include <vector>
+
+#include "sdv_device.cuh"
+#include "sdv_host.h"
+
+namespace sdv {
+
+// ---------------------------------------------------------------- block reduce
+template <int NT>
+__device__ __forceinline__ float2 block_sum2(float a, float b) {
+  __shared__ float2 red[NT / 32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, o);
+    b += __shfl_xor_sync(0xffffffffu, b, o);
+  }
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[w] = make_float2(a, b);
+  __syncthreads();
+  float2 r = make_float2(0.f, 0.f);
+  if (w == 0) {
+    r = (lane < NT / 32) ? red[lane] : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      r.x += __shfl_xor_sync(0xffffffffu, r.x, o);
+      r.y += __shfl_xor_sync(0xffffffffu, r.y, o);
+    }
+  }
+  return r;  // valid in thread 0
+}
+
+// ---------------------------------------------------------------- 16-byte vectors
+__device__ __forceinline__ void unpack(const uint4& v, float (&f)[4]) {
+  f[0] = __uint_as_float(v.x);
+  f[1] = __uint_as_float(v.y);
+  f[2] = __uint_as_float(v.z);
+  f[3] = __uint_as_float(v.w);
+}
+__device__ __forceinline__ void unpack(const uint4& v, float (&f)[8]) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
+}
+
+__device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
+  uint4 r;
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+// ---------------------------------------------------------------- K1
+template <typename T, bool VEC, int VPT>
+__global__ void __launch_bounds__(kK1Threads)
+k_ratio_partials(const T* __restrict__ x, const T* __restrict__ mq, const T* __restrict__ mp,
+                 int L, int64_t d, int C, int64_t chunk, const int32_t* __restrict__ L_eff,
+                 float2* __restrict__ part) {
+  const int64_t tile = blockIdx.x;
+  const int64_t r = tile / C;
+  const int c = (int)(tile - r * C);
+  const int b = (int)(r / L), j = (int)(r - (int64_t)b * L);
+  if (L_eff != nullptr && j >= L_eff[b]) return;
+  const int64_t e0 = (int64_t)c * chunk;
+  const int64_t e1 = min(e0 + chunk, d);
+  const int64_t base = r * d;
+  float s1 = 0.f, s2 = 0.f;
+  if (VEC) {
+    constexpr int V = 16 / (int)sizeof(T);
+    const int64_t v0 = (base + e0) / V;
+    const int nv = (int)((e1 - e0) / V);
+    const uint4* X = reinterpret_cast<const uint4*>(x) + v0;
+    const uint4* Q = reinterpret_cast<const uint4*>(mq) + v0;
+    const uint4* P = reinterpret_cast<const uint4*>(mp) + v0;
+#pragma unroll 1
+    for (int v = threadIdx.x; v < nv; v += kK1Threads * VPT) {
+      uint4 bx[VPT], bq[VPT], bp[VPT];
+      if (v + (VPT - 1) * kK1Threads < nv) {
+        // full sweep: issue all 3 * VPT 16-byte loads before any use
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bx[u] = ldg_stream(X + v + u * kK1Threads);
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bq[u] = ldg_stream(Q + v + u * kK1Threads);
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bp[u] = ldg_stream(P + v + u * kK1Threads);
+      } else {
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) {
+          const int vv = v + u * kK1Threads;
+          const bool ok = vv < nv;
+          bx[u] = ok ? ldg_stream(X + vv) : make_uint4(0u, 0u, 0u, 0u);
+          bq[u] = ok ? ldg_stream(Q + vv) : make_uint4(0u, 0u, 0u, 0u);
+          bp[u] = ok ? ldg_stream(P + vv) : make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < VPT; ++u) {
+        float fx[V], fq[V], fp[V];
+        unpack(bx[u], fx);
+        unpack(bq[u], fq);
+        unpack(bp[u], fp);
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+          const float dl = fp[k] - fq[k];   // m^p - m^q
+          const float a = fx[k] - fp[k];    // yhat - m^p
+          s1 = fmaf(a, dl, s1);
+          s2 = fmaf(dl, dl, s2);
+        }
+      }
+    }
+  } else {
+    for (int64_t e = e0 + threadIdx.x; e < e1; e += kK1Threads) {
+      const float fx = Elem<T>::load(x + base + e);
+      const float fq = Elem<T>::load(mq + base + e);
+      const float fp = Elem<T>::load(mp + base + e);
+      const float dl = fp - fq, a = fx - fp;
+      s1 = fmaf(a, dl, s1);
+      s2 = fmaf(dl, dl, s2);
+    }
+  }
+  const float2 t = block_sum2<kK1Threads>(s1, s2);
+  if (threadIdx.x == 0) part[tile] = t;
+}
+
+// ---------------------------------------------------------------- K2
+__device__ __forceinline__ float warp_incl_sum(float v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += t;
+  }
+  return v;
+}
+__device__ __forceinline__ float warp_incl_max(float v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v = fmaxf(v, t);
+  }
+  return v;
+}
+
+__global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (kK2Threads / 32) + (threadIdx.x >> 5);
+  if (b >= A.B) return;  // warp-uniform
+  const int L = A.L;
+  // window length gamma_k, clamped to [0, L] (device data the host cannot check)
+  const int g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
+  if (g <= 0) {
+    if (lane == 0) {
+      if (A.accepted_len) A.accepted_len[b] = 0;
+      if (A.tau_out) A.tau_out[b] = 0;
+      if (A.state) A.state[b] = ChainState{0, -1, NAN, 0.f, 0.f, 0.f, 0.f, 0u, kKindInactive, 0};
+    }
+    if (A.ell_out)
+      for (int j = lane; j < L; j += 32) A.ell_out[(int64_t)b * L + j] = 0.f;
+    if (A.dn_out)
+      for (int j = lane; j < L; j += 32) A.dn_out[(int64_t)b * L + j] = 0.f;
+    return;
+  }
+  const int nseg = (L + 31) >> 5;
+  float ell[2], dn[2], S1[2], S2[2], sg[2];
+  bool bad = false;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int j = lane + 32 * q;
+    ell[q] = 0.f; dn[q] = 0.f; S1[q] = 0.f; S2[q] = 0.f; sg[q] = 1.f;
+    if (q < nseg && j < g) {
+      if (A.part) {
+        const float2* p = A.part + ((int64_t)b * L + j) * A.C;
+        float a1 = 0.f, a2 = 0.f;
+        for (int c = 0; c < A.C; ++c) {
+          const float2 t = p[c];
+          a1 += t.x;
+          a2 += t.y;
+        }
+        const float s = A.sigma[(int64_t)b * A.sstride + j];
+        S1[q] = a1; S2[q] = a2; sg[q] = s;
+        ell[q] = -(a1 + 0.5f * a2) / (s * s);
+        dn[q] = sqrtf(a2) / s;
+        if (!(s > 0.f) || !isfinite(s)) bad = true;
+      } else {
+        ell[q] = A.ell_in[(int64_t)b * L + j];
+        dn[q] = A.dn_in[(int64_t)b * L + j];
+      }
+      if (!isfinite(ell[q]) || !isfinite(dn[q])) bad = true;
+    }
+    if (q < nseg && j < L) {
+      if (A.ell_out) A.ell_out[(int64_t)b * L + j] = ell[q];
+      if (A.dn_out) A.dn_out[(int64_t)b * L + j] = dn[q];
+    }
+  }
+  const bool any_bad = __any_sync(FULL, bad);
+  if (A.ratios_only) return;
+
+  // coins: eta_j from Philox (b, j, 0, 0), word 0, compared in log space
+  float leta[2];
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int j = lane + 32 * q;
+    leta[q] = 0.f;
+    if (q < nseg && j < g)
+      leta[q] = log_uniform(philox_block(A.seed, (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
+  }
+  float ellw[2] = {ell[0] * A.inv_omega2, ell[1] * A.inv_omega2};
+
+  int tau;            // 1-based
+  float la_res = 0.f; // log alpha_{tau-1}
+  if (A.mode == 0) {
+    // sample verification: c_j = [eta_j < min{1, e^ell_j}]; tau = first failure
+    unsigned fm[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int j = lane + 32 * q;
+      const bool fail = (q < nseg && j < g) && !(leta[q] < fminf(0.f, ellw[q]));
+      fm[q] = __ballot_sync(FULL, fail);
+    }
+    tau = fm[0] ? __ffs(fm[0]) : (fm[1] ? 32 + __ffs(fm[1]) : g + 1);
+  } else {
+    // block verification: log alpha_j = P_j - max(0, max_{m<=j} P_m), P = prefix sums of ell
+    float la[2];
+    float carryP = 0.f, carryM = 0.f;
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int j = lane + 32 * q;
+      const float v = (q < nseg && j < g) ? ellw[q] : 0.f;
+      float P = warp_incl_sum(v, lane) + carryP;
+      float M = fmaxf(warp_incl_max(P, lane), carryM);
+      M = fmaxf(M, 0.f);
+      la[q] = fminf(P - M, 0.f);
+      carryP = __shfl_sync(FULL, P, 31);
+      carryM = __shfl_sync(FULL, M, 31);
+    }
+    // h_j (0-based j): uses |Delta_{j+2}| in paper numbering = dn at j+1
+    const float dn_next0 = __shfl_down_sync(FULL, dn[0], 1);
+    const float dn_first1 = __shfl_sync(FULL, dn[1], 0);
+    const float dn_next1 = __shfl_down_sync(FULL, dn[1], 1);
+    unsigned sm[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int j = lane + 32 * q;
+      bool succ = false;
+      if (q < nseg && j < g) {
+        float lh;
+        if (j == g - 1) {
+          lh = la[q];                                     // h_gamma = alpha_gamma
+        } else {
+          const float Dn = (q == 0) ? (lane == 31 ? dn_first1 : dn_next0) : dn_next1;
+          lh = block_log_h(la[q], Dn);
+        }
+        succ = leta[q] < lh;
+      }
+      sm[q] = __ballot_sync(FULL, succ);
+    }
+    int last = -1;  // 0-based index of the last success
+    if (sm[1]) last = 32 + 31 - __clz(sm[1]);
+    else if (sm[0]) last = 31 - __clz(sm[0]);
+    tau = last + 2;
+    if (tau >= 2) {
+      const int k = tau - 2;
+      const float v0 = __shfl_sync(FULL, la[0], k & 31);
+      const float v1 = __shfl_sync(FULL, la[1], k & 31);
+      la_res = (k < 32) ? v0 : v1;
+    }
+  }
+
+  // quantities of step tau (0-based row tau-1) when a residual is drawn
+  const bool resid = tau <= g;
+  const int rrow = resid ? tau - 1 : 0;
+  const int rq = rrow >> 5, rl = rrow & 31;
+  const float Dt = rq ? __shfl_sync(FULL, dn[1], rl) : __shfl_sync(FULL, dn[0], rl);
+  const float st = rq ? __shfl_sync(FULL, sg[1], rl) : __shfl_sync(FULL, sg[0], rl);
+  const float S1t = rq ? __shfl_sync(FULL, S1[1], rl) : __shfl_sync(FULL, S1[0], rl);
+  const float S2t = rq ? __shfl_sync(FULL, S2[1], rl) : __shfl_sync(FULL, S2[0], rl);
+
+  uint32_t status = any_bad ? 2u : 0u;
+  float U = NAN;
+  int kind;
+  if (!resid) {
+    kind = A.has_bonus ? kKindBonus : kKindCopy;
+  } else if (!(S2t > 0.f) || !(Dt > 0.f)) {
+    kind = kKindZeroDelta;
+    status |= 1u;
+  } else if (A.residual_kind == 1) {
+    kind = kKindReflect;
+  } else {
+    kind = kKindResid;
+    if (A.state) {
+      const uint32_t wbits = philox_block(A.seed, (uint32_t)b, 0u, kStreamUSample, 0u).x;
+      U = usample_warp(Dt, fminf(la_res, 0.f), wbits, &status);
+    }
+  }
+  if (lane == 0) {
+    if (A.accepted_len) A.accepted_len[b] = tau - 1;
+    if (A.tau_out) A.tau_out[b] = tau;
+    if (A.la_res_out) A.la_res_out[b] = la_res;
+    if (A.status_out) A.status_out[b] = status;
+    if (A.aux_out) {
+      float* a = A.aux_out + 4 * (int64_t)b;
+      a[0] = U;
+      a[1] = la_res;
+      a[2] = resid ? Dt : NAN;
+      a[3] = resid ? st : NAN;
+    }
+    if (A.state) {
+      ChainState cs;
+      cs.tau = tau;
+      cs.row = resid ? rrow : g - 1;
+      cs.U = U;
+      cs.la_res = la_res;
+      cs.sigma = st;
+      cs.inv_norm = (S2t > 0.f) ? rsqrtf(S2t) : 0.f;
+      cs.refl = (S2t > 0.f) ? 1.0f + 2.0f * S1t / S2t : 0.f;
+      cs.status = status;
+      cs.kind = kind;
+      cs.pad = 0;
+      A.state[b] = cs;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- K4a / K4b
+template <typename T, bool VEC4>
+__device__ __forceinline__ void load4(const T* p, int64_t i, int64_t d, float (&f)[4]) {
+  if (VEC4 && i + 4 <= d) {
+    if (sizeof(T) == 4) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(p + i));
+      f[0] = v.x; f[1] = v.y; f[2] = v.z; f[3] = v.w;
+    } else {
+      const uint2 v = __ldg(reinterpret_cast<const uint2*>(p + i));
+      f[0] = __uint_as_float(v.x << 16); f[1] = __uint_as_float(v.x & 0xffff0000u);
+      f[2] = __uint_as_float(v.y << 16); f[3] = __uint_as_float(v.y & 0xffff0000u);
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) f[k] = (i + k < d) ? Elem<T>::load(p + i + k) : 0.f;
+  }
+}
+
+template <typename T, bool VEC4>
+__device__ __forceinline__ void store4(T* p, int64_t i, int64_t d, const float (&f)[4]) {
+  if (VEC4 && i + 4 <= d) {
+    if (sizeof(T) == 4) {
+      *reinterpret_cast<float4*>(p + i) = make_float4(f[0], f[1], f[2], f[3]);
+    } else {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(f[0], f[1]);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(f[2], f[3]);
+      uint2 v;
+      memcpy(&v.x, &lo, 4);
+      memcpy(&v.y, &hi, 4);
+      *reinterpret_cast<uint2*>(p + i) = v;
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (i + k < d) Elem<T>::store(p + i + k, f[k]);
+  }
+}
+
+template <typename T, bool VEC4>
+__global__ void __launch_bounds__(kK4Threads)
+k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d, int C4,
+            uint64_t seed, const ChainState* __restrict__ state, float* __restrict__ part4) {
+  const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
+  const ChainState cs = state[b];
+  if (cs.kind != kKindResid) return;
+  const int64_t base = ((int64_t)b * L + cs.row) * d;
+  const int64_t g0 = (int64_t)c * (kK4Chunk / 4);
+  const int64_t g1 = min(g0 + kK4Chunk / 4, (d + 3) / 4);
+  float s = 0.f;
+  for (int64_t gi = g0 + threadIdx.x; gi < g1; gi += kK4Threads) {
+    float fq[4], fp[4];
+    load4<T, VEC4>(mq + base, 4 * gi, d, fq);
+    load4<T, VEC4>(mp + base, 4 * gi, d, fp);
+    const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+    const float g[4] = {G.x, G.y, G.z, G.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) s = fmaf(fp[k] - fq[k], g[k], s);   // tail lanes load 0
+  }
+  const float2 t = block_sum2<kK4Threads>(s, 0.f);
+  if (threadIdx.x == 0) part4[blockIdx.x] = t.x;
+}
+
+template <typename T, bool VEC4>
+__global__ void __launch_bounds__(kK4Threads)
+k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __restrict__ mp,
+              const T* __restrict__ mq_bonus, const float* __restrict__ sigma_bonus, int L,
+              int64_t d, int C4, uint64_t seed, const ChainState* __restrict__ state,
+              const float* __restrict__ part4, T* __restrict__ y) {
+  const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
+  const ChainState cs = state[b];
+  if (cs.kind == kKindInactive) return;
+  const int64_t rbase = ((int64_t)b * L + cs.row) * d;
+  const int64_t ybase = (int64_t)b * d;
+  const int64_t g0 = (int64_t)c * (kK4Chunk / 4);
+  const int64_t g1 = min(g0 + kK4Chunk / 4, (d + 3) / 4);
+  float coef = 0.f;  // U - e^T G for the decomposition residual
+  if (cs.kind == kKindResid) {
+    float T2 = 0.f;
+    for (int k = 0; k < C4; ++k) T2 += part4[(int64_t)b * C4 + k];
+    coef = cs.U - T2 * cs.inv_norm;
+  }
+  for (int64_t gi = g0 + threadIdx.x; gi < g1; gi += kK4Threads) {
+    const int64_t i = 4 * gi;
+    float out[4];
+    if (cs.kind == kKindResid) {
+      float fq[4], fp[4];
+      load4<T, VEC4>(mq + rbase, i, d, fq);
+      load4<T, VEC4>(mp + rbase, i, d, fp);
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      const float g[4] = {G.x, G.y, G.z, G.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float e = (fp[k] - fq[k]) * cs.inv_norm;
+        out[k] = fq[k] + cs.sigma * fmaf(e, coef, g[k]);   // m^q + sigma (G + e (U - e^T G))
+      }
+    } else if (cs.kind == kKindReflect) {
+      float fx[4], fq[4], fp[4];
+      load4<T, VEC4>(x + rbase, i, d, fx);
+      load4<T, VEC4>(mq + rbase, i, d, fq);
+      load4<T, VEC4>(mp + rbase, i, d, fp);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) out[k] = fx[k] - (fp[k] - fq[k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
+    } else if (cs.kind == kKindZeroDelta) {
+      float fq[4];
+      load4<T, VEC4>(mq + rbase, i, d, fq);
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      out[0] = fq[0] + cs.sigma * G.x; out[1] = fq[1] + cs.sigma * G.y;
+      out[2] = fq[2] + cs.sigma * G.z; out[3] = fq[3] + cs.sigma * G.w;
+    } else if (cs.kind == kKindBonus) {
+      float fb[4];
+      load4<T, VEC4>(mq_bonus + ybase, i, d, fb);
+      const float sb = sigma_bonus[b];
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamBonus, 0u);
+      out[0] = fb[0] + sb * G.x; out[1] = fb[1] + sb * G.y;
+      out[2] = fb[2] + sb * G.z; out[3] = fb[3] + sb * G.w;
+    } else {  // copy the last accepted draft
+      load4<T, VEC4>(x + rbase, i, d, out);
+    }
+    store4<T, VEC4>(y + ybase, i, d, out);
+  }
+}
+
+// ---------------------------------------------------------------- stand-alone pieces
+__global__ void __launch_bounds__(128)
+k_usample(const float* __restrict__ D, const float* __restrict__ la, const uint32_t* __restrict__ w,
+          int n, float* __restrict__ U, uint32_t* __restrict__ st) {
+  const int i = blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (i >= n) return;  // warp-uniform
+  const float Dn = D[i];
+  float l = la[i];
+  uint32_t status = 0u;
+  float u = NAN;
+  if (isnan(Dn) || isnan(l)) {
+    status = 2u;
+  } else if (!(Dn > 0.f) || isinf(Dn)) {
+    status = 1u;
+  } else {
+    l = fminf(l, 0.f);
+    u = usample_warp(Dn, l, w[i], &status);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    U[i] = u;
+    if (st) st[i] = status;
+  }
+}
+
+__global__ void k_philox(const uint4* __restrict__ ctr, uint64_t seed, int n, uint4* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) out[i] = philox4x32_10(ctr[i], (uint32_t)seed, (uint32_t)(seed >> 32));
+}
+
+__global__ void k_normals(uint64_t seed, int B, int64_t d, uint32_t stream, uint32_t sub, float* out) {
+  const int64_t ng = (d + 3) / 4;
+  const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= (int64_t)B * ng) return;
+  const int b = (int)(t / ng);
+  const int64_t gi = t - (int64_t)b * ng;
+  const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, stream, sub);
+  const float g[4] = {G.x, G.y, G.z, G.w};
+  for (int k = 0; k < 4; ++k)
+    if (4 * gi + k < d) out[(int64_t)b * d + 4 * gi + k] = g[k];
+}
+
+// ---------------------------------------------------------------- host side
+static thread_local int g_last_cuda_error = 0;
+
+static int check_launch() {
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    g_last_cuda_error = (int)e;
+    return SDV_ECUDA;
+  }
+  return SDV_OK;
+}
+
+static bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ---- per-thread timing ring (sdv_timing_enable / sdv_timing_read).  Records use
+// cudaEventRecordExternal so that, under stream capture, they become event-record
+// nodes of the graph (a plain record there only expresses a dependency).
+struct TimingRing {
+  std::vector<cudaEvent_t> ev;  // slots x 4
+  int slots = 0;
+  long long next = 0;
+};
+static thread_local TimingRing g_timing;
+
+static void timing_destroy() {
+  for (cudaEvent_t e : g_timing.ev) cudaEventDestroy(e);
+  g_timing.ev.clear();
+  g_timing.slots = 0;
+  g_timing.next = 0;
+}
+
+static cudaEvent_t* timing_slot() {
+  if (g_timing.slots == 0) return nullptr;
+  const int s = (int)(g_timing.next % g_timing.slots);
+  ++g_timing.next;
+  return &g_timing.ev[4 * (size_t)s];
+}
+
+WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
+  WsLayout w{};
+  const int es = dtype == SDV_BF16 ? 2 : 4;
+  // vectors per thread: the smallest sweep that covers a row, capped at kK1Vpt,
+  // so that common row lengths run whole, unguarded sweeps
+  const int64_t vec_per_row = (d * es + 15) / 16;
+  w.vpt1 = (int)std::min<int64_t>(kK1Vpt, std::max<int64_t>(1, (vec_per_row + kK1Threads - 1) / kK1Threads));
+  w.chunk1 = (int64_t)kK1Threads * w.vpt1 * (16 / es);
+  w.C1 = (int)((d + w.chunk1 - 1) / w.chunk1);
+  w.C4 = (int)((d + kK4Chunk - 1) / kK4Chunk);
+  auto up = [](size_t v) { return (v + 255) & ~(size_t)255; };
+  size_t off = 0;
+  w.part_off = off;
+  off = up(off + sizeof(float2) * (size_t)B * L * w.C1);
+  w.state_off = off;
+  off = up(off + sizeof(ChainState) * (size_t)B);
+  w.part4_off = off;
+  off = up(off + sizeof(float) * (size_t)B * w.C4);
+  w.total = off;
+  return w;
+}
+
+static int validate_window(const void* x, const void* mq, const void* mp, const float* sigma,
+                           int64_t sstride, int B, int L, int64_t d, int dtype) {
+  if (!x || !mq || !mp || !sigma) return SDV_EINVAL;
+  if (B < 1 || L < 1 || L > SDV_MAX_L || d < 1) return SDV_EINVAL;
+  if (dtype != SDV_F32 && dtype != SDV_BF16) return SDV_EINVAL;
+  if (sstride < 0) return SDV_EINVAL;
+  if ((double)B * L * (double)d > 9.0e18) return SDV_EINVAL;
+  if (B > (1 << 30)) return SDV_EINVAL;
+  const size_t es = dtype == SDV_BF16 ? 2 : 4;
+  if (!aligned(x, es) || !aligned(mq, es) || !aligned(mp, es) || !aligned(sigma, 4)) return SDV_EALIGN;
+  return SDV_OK;
+}
+
+template <typename T>
+static void launch_k1(const void* x, const void* mq, const void* mp, int B, int L, int64_t d,
+                      const int32_t* L_eff, const WsLayout& w, float2* part, cudaStream_t s) {
+  constexpr int V = 16 / (int)sizeof(T);
+  const bool vec = (d % V == 0) && aligned(x, 16) && aligned(mq, 16) && aligned(mp, 16);
+  const unsigned tiles = (unsigned)((int64_t)B * L * w.C1);
+  const T *X = (const T*)x, *Q = (const T*)mq, *P = (const T*)mp;
+  if (!vec) {
+    k_ratio_partials<T, false, 1><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part);
+    return;
+  }
+  switch (w.vpt1) {
+    case 1: k_ratio_partials<T, true, 1><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
+    case 2: k_ratio_partials<T, true, 2><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
+    case 3: k_ratio_partials<T, true, 3><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
+    default: k_ratio_partials<T, true, 4><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
+  }
+}
+
+template <typename T>
+static void launch_k4(const void* x, const void* mq, const void* mp, const void* mqb,
+                      const float* sb, int B, int L, int64_t d, uint64_t seed, const WsLayout& w,
+                      const ChainState* st, float* part4, void* y, cudaStream_t s) {
+  const bool vec = (d % 4 == 0) && aligned(x, 4 * sizeof(T)) && aligned(mq, 4 * sizeof(T)) &&
+                   aligned(mp, 4 * sizeof(T)) && aligned(y, 4 * sizeof(T)) &&
+                   (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
+  const unsigned grid = (unsigned)((int64_t)B * w.C4);
+  if (vec) {
+    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, st, part4);
+    k_resid_write<T, true><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
+                                                      (const T*)mqb, sb, L, d, w.C4, seed, st, part4, (T*)y);
+  } else {
+    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, st, part4);
+    k_resid_write<T, false><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
+                                                       (const T*)mqb, sb, L, d, w.C4, seed, st, part4, (T*)y);
+  }
+}
+
+}  // namespace sdv
+
+using namespace sdv;
+
+extern "C" {
+
+const char* sdv_version(void) { return "specdiff-gb300 0.1 (sm_103a)"; }
+
+const char* sdv_strerror(int code) {
+  switch (code) {
+    case SDV_OK: return "ok";
+    case SDV_EINVAL: return "invalid argument";
+    case SDV_EALIGN: return "misaligned pointer";
+    case SDV_ECUDA: return "CUDA launch failure";
+    case SDV_ENOWORKSPACE: return "workspace missing or too small";
+    default: return "unknown error";
+  }
+}
+
+int sdv_last_cuda_error(void) { return g_last_cuda_error; }
+
+size_t sdv_workspace_bytes(int B, int L, int64_t d, int dtype) {
+  if (B < 1 || L < 1 || L > SDV_MAX_L || d < 1 || (dtype != SDV_F32 && dtype != SDV_BF16)) return 0;
+  return ws_layout(B, L, d, dtype).total;
+}
+
+int sdv_verify_ex(const void* x_draft, const void* mu_target, const void* mu_draft,
+                  const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                  uint64_t seed, int mode, const int32_t* L_eff, const void* mu_target_bonus,
+                  const float* sigma_bonus, int residual_kind, float omega,
+                  int32_t* accepted_len, void* y_out, float* log_ratio_out,
+                  float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
+                  void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
+  if (rc != SDV_OK) return rc;
+  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
+  if (residual_kind != SDV_RESIDUAL_DECOMPOSITION && residual_kind != SDV_RESIDUAL_REFLECTION)
+    return SDV_EINVAL;
+  if (residual_kind == SDV_RESIDUAL_REFLECTION && mode != SDV_MODE_SAMPLE) return SDV_EINVAL;
+  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
+  if (!accepted_len || !y_out) return SDV_EINVAL;
+  if ((mu_target_bonus == nullptr) != (sigma_bonus == nullptr)) return SDV_EINVAL;
+  const size_t es = dtype == SDV_BF16 ? 2 : 4;
+  if (!aligned(y_out, es) || !aligned(accepted_len, 4) ||
+      (mu_target_bonus && !aligned(mu_target_bonus, es)) || (sigma_bonus && !aligned(sigma_bonus, 4)) ||
+      (L_eff && !aligned(L_eff, 4)) || (log_ratio_out && !aligned(log_ratio_out, 4)) ||
+      (delta_norm_out && !aligned(delta_norm_out, 4)) || (status_out && !aligned(status_out, 4)) ||
+      (chain_aux_out && !aligned(chain_aux_out, 4)))
+    return SDV_EALIGN;
+  const WsLayout w = ws_layout(B, L, d, dtype);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if (!aligned(workspace, 256)) return SDV_EALIGN;
+  cudaStream_t s = (cudaStream_t)stream;
+  char* ws = (char*)workspace;
+  float2* part = (float2*)(ws + w.part_off);
+  ChainState* st = (ChainState*)(ws + w.state_off);
+  float* part4 = (float*)(ws + w.part4_off);
+
+  cudaEvent_t* tev = timing_slot();
+  if (tev) cudaEventRecordWithFlags(tev[0], s, cudaEventRecordExternal);
+  if (dtype == SDV_F32) launch_k1<float>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
+  else launch_k1<__nv_bfloat16>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
+  if ((rc = check_launch()) != SDV_OK) return rc;
+  if (tev) cudaEventRecordWithFlags(tev[1], s, cudaEventRecordExternal);
+
+  ScanArgs A{};
+  A.part = part; A.C = w.C1; A.sigma = sigma; A.sstride = sigma_stride_b;
+  A.B = B; A.L = L; A.L_eff = L_eff; A.seed = seed; A.mode = mode;
+  A.inv_omega2 = 1.0f / (omega * omega); A.residual_kind = residual_kind;
+  A.has_bonus = mu_target_bonus != nullptr; A.ratios_only = false;
+  A.ell_out = log_ratio_out; A.dn_out = delta_norm_out; A.accepted_len = accepted_len;
+  A.status_out = status_out; A.aux_out = chain_aux_out; A.state = st;
+  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, s>>>(A);
+  if ((rc = check_launch()) != SDV_OK) return rc;
+  if (tev) cudaEventRecordWithFlags(tev[2], s, cudaEventRecordExternal);
+
+  if (dtype == SDV_F32)
+    launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, st, part4, y_out, s);
+  else
+    launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, st, part4, y_out, s);
+  rc = check_launch();
+  if (tev) cudaEventRecordWithFlags(tev[3], s, cudaEventRecordExternal);
+  return rc;
+}
+
+int sdv_timing_enable(int slots) {
+  if (slots < 0 || slots > (1 << 20)) return SDV_EINVAL;
+  timing_destroy();
+  if (slots == 0) return SDV_OK;
+  g_timing.ev.resize(4 * (size_t)slots);
+  for (auto& e : g_timing.ev) {
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      g_last_cuda_error = (int)cudaGetLastError();
+      g_timing.ev.clear();
+      return SDV_ECUDA;
+    }
+  }
+  g_timing.slots = slots;
+  return SDV_OK;
+}
+
+int sdv_timing_read(int n_calls, float* ms3) {
+  if (!ms3 || g_timing.slots == 0 || n_calls < 1 || n_calls > g_timing.slots ||
+      n_calls > g_timing.next)
+    return SDV_EINVAL;
+  double acc[3] = {0, 0, 0};
+  for (int i = 0; i < n_calls; ++i) {
+    const int s = (int)((g_timing.next - 1 - i) % g_timing.slots);
+    cudaEvent_t* e = &g_timing.ev[4 * (size_t)s];
+    if (cudaEventSynchronize(e[3]) != cudaSuccess) {
+      g_last_cuda_error = (int)cudaGetLastError();
+      return SDV_ECUDA;
+    }
+    for (int k = 0; k < 3; ++k) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, e[k], e[k + 1]) != cudaSuccess) {
+        g_last_cuda_error = (int)cudaGetLastError();
+        return SDV_ECUDA;
+      }
+      acc[k] += ms;
+    }
+  }
+  for (int k = 0; k < 3; ++k) ms3[k] = (float)acc[k];
+  return SDV_OK;
+}
+
+int sdv_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
+               const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+               uint64_t seed, int mode, int32_t* accepted_len, void* y_out,
+               float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
+               void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  return sdv_verify_ex(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                       mode, nullptr, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION, 1.0f,
+                       accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, nullptr,
+                       workspace, workspace_bytes, stream);
+}
+
+int sdv_log_ratios(const void* x_draft, const void* mu_target, const void* mu_draft,
+                   const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                   const int32_t* L_eff, float* log_ratio_out, float* delta_norm_out,
+                   void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
+  if (rc != SDV_OK) return rc;
+  if (!log_ratio_out || !delta_norm_out) return SDV_EINVAL;
+  if (!aligned(log_ratio_out, 4) || !aligned(delta_norm_out, 4) || (L_eff && !aligned(L_eff, 4)))
+    return SDV_EALIGN;
+  const WsLayout w = ws_layout(B, L, d, dtype);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if (!aligned(workspace, 256)) return SDV_EALIGN;
+  cudaStream_t s = (cudaStream_t)stream;
+  float2* part = (float2*)((char*)workspace + w.part_off);
+  if (dtype == SDV_F32) launch_k1<float>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
+  else launch_k1<__nv_bfloat16>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
+  if ((rc = check_launch()) != SDV_OK) return rc;
+  ScanArgs A{};
+  A.part = part; A.C = w.C1; A.sigma = sigma; A.sstride = sigma_stride_b;
+  A.B = B; A.L = L; A.L_eff = L_eff; A.inv_omega2 = 1.f; A.ratios_only = true;
+  A.ell_out = log_ratio_out; A.dn_out = delta_norm_out;
+  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, s>>>(A);
+  return check_launch();
+}
+
+int sdv_accept_scan(const float* log_ratio, const float* delta_norm, int B, int L,
+                    const int32_t* L_eff, uint64_t seed, int mode, float omega, int32_t* tau_out,
+                    float* log_alpha_res_out, sdv_stream_t stream) {
+  if (!log_ratio || !delta_norm || !tau_out) return SDV_EINVAL;
+  if (B < 1 || L < 1 || L > SDV_MAX_L || B > (1 << 30)) return SDV_EINVAL;
+  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
+  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
+  if (!aligned(log_ratio, 4) || !aligned(delta_norm, 4) || !aligned(tau_out, 4) ||
+      (log_alpha_res_out && !aligned(log_alpha_res_out, 4)) || (L_eff && !aligned(L_eff, 4)))
+    return SDV_EALIGN;
+  ScanArgs A{};
+  A.ell_in = log_ratio; A.dn_in = delta_norm; A.B = B; A.L = L; A.L_eff = L_eff;
+  A.seed = seed; A.mode = mode; A.inv_omega2 = 1.0f / (omega * omega);
+  A.tau_out = tau_out; A.la_res_out = log_alpha_res_out;
+  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, (cudaStream_t)stream>>>(A);
+  return check_launch();
+}
+
+int sdv_usample(const float* delta_norm, const float* log_alpha, const uint32_t* w_bits, int n,
+                float* U_out, uint32_t* status_out, sdv_stream_t stream) {
+  if (!delta_norm || !log_alpha || !w_bits || !U_out || n < 0) return SDV_EINVAL;
+  if (!aligned(delta_norm, 4) || !aligned(log_alpha, 4) || !aligned(w_bits, 4) ||
+      !aligned(U_out, 4) || (status_out && !aligned(status_out, 4)))
+    return SDV_EALIGN;
+  if (n == 0) return SDV_OK;
+  k_usample<<<(n + 3) / 4, 128, 0, (cudaStream_t)stream>>>(delta_norm, log_alpha, w_bits, n, U_out, status_out);
+  return check_launch();
+}
+
+int sdv_philox(const uint32_t* ctr, uint64_t seed, int n, uint32_t* out, sdv_stream_t stream) {
+  if (!ctr || !out || n < 0) return SDV_EINVAL;
+  if (!aligned(ctr, 16) || !aligned(out, 16)) return SDV_EALIGN;
+  if (n == 0) return SDV_OK;
+  k_philox<<<(n + 255) / 256, 256, 0, (cudaStream_t)stream>>>((const uint4*)ctr, seed, n, (uint4*)out);
+  return check_launch();
+}
+
+int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub, float* out,
+                sdv_stream_t stream) {
+  if (!out || B < 1 || d < 1 || stream_id < 0) return SDV_EINVAL;
+  if (!aligned(out, 4)) return SDV_EALIGN;
+  const int64_t n = (int64_t)B * ((d + 3) / 4);
+  k_normals<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(seed, B, d, (uint32_t)stream_id, sub, out);
+  return check_launch();
+}
+
+}  // extern "C"

@@ -1,0 +1,96 @@
+"""Shared helpers of the GPU parity tests: move seeded inputs to the device, run the
+C-ABI path and the oracle on the same inputs, and compare with the stated tolerances.
+
+Tolerances (from the verification step's accuracy targets):
+  * log ratios and |Delta|: |gpu - oracle| <= 1e-5 * max(1, |oracle|);
+  * accepted lengths: bit-exact, except for a chain whose oracle run has a coin
+    within the tie band of its threshold: |log eta_j - log thr_j| < 1e-4 plus the
+    propagated log-ratio tolerance (thr = min{1, e^ell} in sample mode, h_j in block
+    mode, where log alpha_j accumulates the tolerance of ell_1..ell_j);
+  * output states (chains with equal tau): 1e-5 absolute for fp32 inputs, 2e-2 for bf16.
+"""
+import numpy as np
+import torch
+
+from oracle import philox as OP
+from oracle import verify as OV
+
+TOL_Y = {"f32": 1e-5, "bf16": 2e-2}
+
+
+def to_dev(inp, name):
+    if inp["dtype"] == "bf16":
+        bits = np.ascontiguousarray(inp[name + "_bits"]).view(np.int16)
+        return torch.from_numpy(bits).cuda().view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(inp[name])).cuda()
+
+
+def run_gpu(api, inp, seed, mode, sigma=None, **kw):
+    x = to_dev(inp, "x_draft")
+    mq = to_dev(inp, "mu_target")
+    mp = to_dev(inp, "mu_draft")
+    sg = torch.from_numpy(np.ascontiguousarray(inp["sigma"] if sigma is None else sigma)).cuda()
+    dev_kw = {}
+    for k, v in kw.items():
+        if isinstance(v, np.ndarray):
+            v = torch.from_numpy(np.ascontiguousarray(v)).cuda()
+        dev_kw[k] = v
+    if "mu_target_bonus" in dev_kw and inp["dtype"] == "bf16":
+        dev_kw["mu_target_bonus"] = dev_kw["mu_target_bonus"].to(torch.bfloat16)
+    r = api.verify(x, mq, mp, sg, seed, mode, with_aux=True, **dev_kw)
+    torch.cuda.synchronize()
+    out = {k: (v.float().cpu().numpy() if v.dtype == torch.bfloat16 else v.cpu().numpy())
+           for k, v in r.items()}
+    return out
+
+
+def near_tie(o, mode, omega=1.0, band=1e-4, rtol=1e-5):
+    """Per chain: does the oracle run have a coin inside the tie band of its threshold?"""
+    ell = o["ell"] / (omega * omega)
+    leta = np.log(o["eta"])
+    slack = rtol * np.maximum(1.0, np.abs(o["ell"])) / (omega * omega)
+    n, L = ell.shape
+    if mode == OV.MODE_SAMPLE:
+        thr = np.minimum(0.0, ell)
+        tie = np.abs(leta - thr) < band + slack
+    else:
+        with np.errstate(divide="ignore"):
+            lh = np.log(o["h"][:, 1:])
+        cum = np.cumsum(slack, axis=1)
+        tie = np.abs(leta - lh) < band + cum
+    return tie.any(axis=1)
+
+
+def compare(g, o, mode, dtype, omega=1.0, max_tie_frac=0.05):
+    """Assert parity of a GPU result dict with an oracle result dict (same chains)."""
+    ell_g, ell_o = g["log_ratio"], o["ell"]
+    assert np.all(np.abs(ell_g - ell_o) <= 1e-5 * np.maximum(1.0, np.abs(ell_o))), \
+        "log ratio max err %g" % np.max(np.abs(ell_g - ell_o) / np.maximum(1.0, np.abs(ell_o)))
+    dn_g, dn_o = g["delta_norm"], o["dnorm"]
+    assert np.all(np.abs(dn_g - dn_o) <= 1e-5 * np.maximum(1.0, dn_o)), "delta norm"
+    acc_g, acc_o = g["accepted_len"], o["accepted_len"]
+    diff = acc_g != acc_o
+    if diff.any():
+        ties = near_tie(o, mode, omega)
+        assert np.all(ties[diff]), "accepted length differs outside the tie band: chains %s" % \
+            np.nonzero(diff & ~ties)[0][:10]
+        assert diff.mean() <= max_tie_frac
+    same = ~diff
+    yg, yo = g["y"][same], o["y"][same]
+    act = np.isfinite(yo).all(axis=1)
+    err = np.abs(yg[act] - yo[act])
+    tol = TOL_Y[dtype]
+    assert err.size == 0 or err.max() <= tol, "y max err %g (tol %g)" % (err.max(), tol)
+    assert np.array_equal(g["status"][same] & 3, o["status"][same] & 3)
+    return int(diff.sum())
+
+
+def oracle_for(inp, seed, mode, chains=None, **kw):
+    return OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], seed,
+                     mode, chains=chains, **kw)
+
+
+def philox_words(ctr, seed):
+    k0, k1 = OP.key_of(seed)
+    w = OP.philox4x32_10(ctr[:, 0], ctr[:, 1], ctr[:, 2], ctr[:, 3], k0, k1)
+    return np.stack(w, axis=1).astype(np.uint32)

@@ -1,7 +1,7 @@
 """Benchmark of the speculative-diffusion verification step on GB300.
 
-One step = one sdv_verify call (log-ratio pass, acceptance scan + residual
-U-draw, residual write) on one batch of the pixel-scale workload (B=256 chains,
+One step = one sdv_verify call (one fused kernel: log-ratio pass, acceptance
+scan, residual U-draw, residual write) on one batch of the pixel-scale workload (B=256 chains,
 L=8 draft steps, d=3x32x32 fp32, block verification) with inputs resident in
 HBM.  Eight input sets (8 x 75.5 MB, well above the 129 MB L2) rotate between
 steps, so every step reads its inputs from HBM.  Steps are captured into CUDA
@@ -9,7 +9,7 @@ graphs and replayed.
 
 Prints ONE JSON line (rank 0):
   value      verified draft-steps/s (B*L per step), whole job
-  roofline   the log-ratio pass (dominant kernel): algorithmic bytes / its mean
+  roofline   the fused verify kernel (dominant kernel): algorithmic bytes / its mean
              duration from CUDA events inside the timed region, vs measured HBM peak
   e2e        the same metric through the public API from pinned host buffers
              (host->device copy of the window, device->host copy of results)
@@ -63,9 +63,9 @@ def peaks():
 
 
 def profile_traffic(kernel_src):
-    """dram bytes per launch of the log-ratio pass from the committed ncu summary, if the
-    kernel source is unchanged since the capture (else None)."""
-    path = os.path.join(ROOT, "profiles", "ratio_partials_pixel.md")
+    """dram bytes per launch of the fused verify kernel from the committed ncu summary, if
+    the kernel source is unchanged since the capture (else None)."""
+    path = os.path.join(ROOT, "profiles", "k_verify_pixel.md")
     if not os.path.exists(path):
         return None
     txt = open(path).read()
@@ -120,6 +120,26 @@ class ClockSampler:
             return None
         return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)),
                 "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def long_rows(d):
+    """Rows longer than 16384 elements get their residual from two extra kernels."""
+    return (d + 3) // 4 > 4096
+
+
+def launches_per_step(d):
+    """Kernels one sdv_verify call launches: the fused verify kernel, plus the
+    residual dot / write kernels for long rows (the ticket reset is a memset)."""
+    return 3 if long_rows(d) else 1
+
+
+def fused_kernel_bytes(B, L, d, dtype):
+    """Algorithmic bytes of the fused kernel per call: x, m^q, m^p read once, and, when it
+    also writes the residual, the rejected row's m^q and m^p (upper bound: every chain)
+    re-read plus y written."""
+    s = W.bytes_per_element(dtype)
+    main = 3 * B * L * d * s
+    return main if long_rows(d) else main + 3 * B * d * s
 
 
 def dist_setup():
@@ -291,7 +311,7 @@ def main():
     ms_total = ev0.elapsed_time(ev1)
     clk = clocks.stop()
     n_timed = G_STEPS if use_graph and args.steps % G_STEPS == 0 else min(args.steps, G_STEPS)
-    k1_ms, k2_ms, k4_ms = (v / n_timed for v in binding.sdv_timing_read(n_timed))
+    kv_ms, kr_ms, _ = (v / n_timed for v in binding.sdv_timing_read(n_timed))
     binding.sdv_timing_enable(0)
     if pg:
         t = torch.tensor([ms_total], device=dev)
@@ -338,8 +358,8 @@ def main():
     d2h = Bn * 4 + Bn * d * hx.element_size()
 
     hbm_peak, peak_kind = peaks()
-    k1_bytes = set_bytes
-    achieved = k1_bytes / (k1_ms * 1e-3) / 1e9
+    kv_bytes = fused_kernel_bytes(Bn, L, d, dt_name)
+    achieved = kv_bytes / (kv_ms * 1e-3) / 1e9
     kernel_src = os.path.join(ROOT, "paper_2606_13426_gb300", "csrc", "sdv_verify.cu")
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -356,15 +376,16 @@ def main():
                    "cuda_graph": use_graph},
         "hbm_gbs_step": (set_bytes / (ms_step * 1e-3)) / 1e9,
         "mean_tau_block": taus["block"], "mean_tau_sample": taus["sample"],
-        "phase_us": {"log_ratio_pass": 1e3 * k1_ms, "scan_usample": 1e3 * k2_ms,
-                     "residual": 1e3 * k4_ms},
+        "phase_us": {"verify_kernel": 1e3 * kv_ms, "long_row_residual": 1e3 * kr_ms},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                     "kernel": "k_ratio_partials (log-ratio pass)",
+                     "kernel": "k_verify (fused: log-ratio pass, acceptance, U-draw%s)"
+                               % ("" if long_rows(d) else ", residual write"),
+                     "algorithmic_bytes": kv_bytes,
                      "traffic": profile_traffic(kernel_src)},
         "e2e": {"value": world * Bn * L / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": launches_per_step(d) * args.steps,
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.skip_cpu:

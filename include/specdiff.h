@@ -204,20 +204,22 @@ int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub,
 /*
  * Profiling aid (not part of the method): when enabled, every later
  * sdv_verify / sdv_verify_ex call made on this host thread records four CUDA
- * events on its stream - before the log-ratio pass, after it, after the
- * acceptance scan, after the residual write - into a ring of `slots` entries.
- * The records are ordinary stream work, so they are captured into a CUDA graph
- * like the kernels.  The events are created here (host objects; no device
- * memory).  slots = 0 disables timing and destroys the events.
+ * events on its stream into a ring of `slots` entries: before the fused
+ * verify kernel, after it, and (twice) after the separate residual kernels
+ * used for rows longer than 16384 elements.  The records are ordinary stream
+ * work, so they are captured into a CUDA graph like the kernels.  The events
+ * are created here (host objects; no device memory).  slots = 0 disables
+ * timing and destroys the events.
  */
 int sdv_timing_enable(int slots);
 
 /*
  * Waits for the events of the last `n_calls` recorded calls (1 <= n_calls <=
  * slots) and writes their summed phase times in milliseconds:
- * ms3[0] log-ratio pass (K1), ms3[1] acceptance scan + U-sampler (K2),
- * ms3[2] residual dot + write (K4).  SDV_EINVAL if timing is off or fewer
- * calls were recorded.
+ * ms3[0] the fused verify kernel (log-ratio pass, acceptance, U-draw and, for
+ * rows up to 16384 elements, the residual write), ms3[1] the long-row residual
+ * kernels (0 otherwise), ms3[2] reserved (0).  SDV_EINVAL if timing is off or
+ * fewer calls were recorded.
  */
 int sdv_timing_read(int n_calls, float *ms3);
 

@@ -11,6 +11,8 @@
 //    Eq. u-cdf, Algorithm u-sample) as a warp-cooperative multisection.
 //
 // Everything is fp32: GB300's fp64 rate is a small fraction of its fp32 rate.
+// The special-function helpers are __noinline__: inlined at every call site they
+// made the acceptance-scan kernel's code too large for the instruction cache.
 // The forms below avoid the cancellations that fp32 would otherwise suffer:
 //  - v = alpha Phi(a+) - Phi(a-) is written as alpha Phi(a+) (1 - e^{x0}) with
 //    x0 = log(Phi(a-)/(alpha Phi(a+))) = g(a-) - g(a+), exact because
@@ -105,34 +107,48 @@ static __constant__ float kGLx[4] = {0.18343464249564978f, 0.52553240991632899f,
 static __constant__ float kGLw[4] = {0.36268378337836166f, 0.31370664587788688f,
                                           0.22238103445337443f, 0.10122853629037706f};
 
-// log Phi(a).
-__device__ __forceinline__ float log_ndtr(float a) {
-  if (a < -1.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf)) - 0.5f * a * a;
+// log Phi(a); for a <= 0 through the scaled complement erfcx (no underflow).
+static __device__ __noinline__ float log_ndtr(float a) {
   if (a > 0.0f) return log1pf(-0.5f * erfcf(a * kSqrtHalf));
-  return logf(0.5f * erfcf(-a * kSqrtHalf));
+  return logf(0.5f * erfcxf(-a * kSqrtHalf)) - 0.5f * a * a;
 }
 
 // g(a) = log Phi(a) + a^2/2 (moderate for a <= 0).
-__device__ __forceinline__ float gfun(float a) {
-  if (a < -1.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf));
+static __device__ __noinline__ float gfun(float a) {
+  if (a <= 0.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf));
   return log_ndtr(a) + 0.5f * a * a;
 }
 
-// g'(s) = lambda(s) + s > 0.
-__device__ __forceinline__ float gprime(float s) {
+// g'(s) = lambda(s) + s > 0.  The continued fraction is evaluated bottom-up with a
+// fast reciprocal: each level adds n/acc << x to x, so the reciprocal's few-ulp
+// error is damped by the levels above; only the final division is exact.  Deeper
+// levels are needed only near the switch point (16 levels give ~5e-10 at x = 4,
+// 8 levels ~4e-10 at x = 8).
+static __device__ __noinline__ float gprime(float s) {
   if (s < -4.0f) {
     const float x = -s;
     float acc = x;
+    if (x < 8.0f) {
 #pragma unroll
-    for (int n = 16; n >= 2; --n) acc = x + (float)n / acc;
+      for (int n = 16; n >= 9; --n) acc = x + __fdividef((float)n, acc);
+    }
+#pragma unroll
+    for (int n = 8; n >= 2; --n) acc = x + __fdividef((float)n, acc);
     return 1.0f / acc;
   }
-  return expf(-0.5f * s * s - kHalfLog2Pi - log_ndtr(s)) + s;
+  // lambda(s) = phi(s)/Phi(s) = sqrt(2/pi) / erfcx(-s/sqrt 2); beyond s = 9 it is < 1e-18
+  if (s > 9.0f) return s;
+  return 0.79788456080286536f / erfcxf(-s * kSqrtHalf) + s;
 }
 
-// g(hi) - g(hi - h) for h >= 0; the interval length is exactly h.
-__device__ __forceinline__ float gdiff(float hi, float h) {
-  if (h <= fmaxf(2.0f, 0.5f * fabsf(hi))) {
+// g(hi) - g(hi - h) for h >= 0; the interval length is exactly h.  The direct
+// difference of two g values is accurate to a few 1e-7 absolute (|g| <= ~3 for
+// arguments above -8); it is replaced by 8-point Gauss-Legendre quadrature of g'
+// where the difference itself is small: short intervals and the deep left tail
+// (g' ~ 1/|s| there).
+static __device__ __noinline__ float gdiff(float hi, float h) {
+  const bool careful = (h < 0.5f) || (hi < -2.0f);
+  if (careful && h <= fmaxf(2.0f, 0.5f * fabsf(hi))) {
     const float r = 0.5f * h, m = hi - r;
     float acc = 0.0f;
 #pragma unroll
@@ -163,7 +179,7 @@ __device__ __forceinline__ float logaddexp(float a, float b) {
 }
 
 // log(Phi(b) - Phi(a)) for a < b.
-__device__ __forceinline__ float log_ndtr_interval(float a, float b) {
+static __device__ __noinline__ float log_ndtr_interval(float a, float b) {
   if (b <= 0.0f) return log_ndtr(b) + log1mexp(log_ndtr(a) - log_ndtr(b));
   if (a >= 0.0f) return log_ndtr(-a) + log1mexp(log_ndtr(-b) - log_ndtr(-a));
   return log1pf(-(expf(log_ndtr(a)) + expf(log_ndtr(-b))));
@@ -172,7 +188,7 @@ __device__ __forceinline__ float log_ndtr_interval(float a, float b) {
 // ---------------------------------------------------------------- block verification
 // log h_j, h_j = v_j / (v_j + 1 - alpha_j), from log alpha_j (<= 0) and |Delta_{j+1}|.
 // Limits: alpha_j = 1 -> h = 1; alpha_j = 0 or |Delta_{j+1}| = 0 (alpha_j < 1) -> h = 0.
-__device__ __forceinline__ float block_log_h(float la, float Dn) {
+static __device__ __noinline__ float block_log_h(float la, float Dn) {
   if (isnan(la) || isnan(Dn)) return -INFINITY;
   if (!(la < 0.0f)) return 0.0f;
   if (la == -INFINITY || !(Dn > 0.0f)) return -INFINITY;
@@ -190,7 +206,7 @@ struct UParams {
   float lvn;  // log v - log phi(a-)
 };
 
-__device__ __forceinline__ UParams usample_setup(float D, float la) {
+static __device__ __noinline__ UParams usample_setup(float D, float la) {
   UParams P;
   P.D = D;
   P.la = la;
@@ -203,7 +219,7 @@ __device__ __forceinline__ UParams usample_setup(float D, float la) {
 }
 
 // log Psi(a+ - t), t > 0.
-__device__ __forceinline__ float usample_log_psi(float t, const UParams& P) {
+static __device__ __noinline__ float usample_log_psi(float t, const UParams& P) {
   const float u = P.ap - t;
   const float x = -gdiff(u, P.D) - P.D * t;     // log(Phi(u - D) / (alpha Phi(u)))
   if (u < 0.0f)
@@ -212,7 +228,7 @@ __device__ __forceinline__ float usample_log_psi(float t, const UParams& P) {
 }
 
 // log(1 - Psi(a+ - t)), t > 0.
-__device__ __forceinline__ float usample_log_1mpsi(float t, const UParams& P) {
+static __device__ __noinline__ float usample_log_1mpsi(float t, const UParams& P) {
   if (P.D * t <= 1.0f && -P.am * t <= 4.0f) {
     const float r = 0.5f * t;
     float acc = 0.0f;
@@ -230,46 +246,83 @@ __device__ __forceinline__ float usample_log_1mpsi(float t, const UParams& P) {
   return lA + log1mexp(lB - lA) - P.lv;
 }
 
-// U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32.  Must be called by all 32
-// lanes of a warp with the same arguments; every lane returns U.
-// In t = a+ - u (Psi decreasing in t): a parallel doubling search over
-// t = 2^-12 .. 2^19 (the paper's bracket growth, all steps at once), then
-// five rounds of 32-way multisection (width / 2^25).  Lower half of w
-// compares log Psi with log w, upper half log(1 - Psi) with log(1 - w).
-__device__ __forceinline__ float usample_warp(float D, float la, uint32_t wbits,
-                                              uint32_t* status) {
+// Shared scratch of usample_block.
+struct USampleScratch {
+  int first[32];
+  float t[2];
+  float g[2];
+};
+
+// U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32, by all NT threads of a CTA (NT a
+// multiple of 32, <= 1024) with the same arguments; every thread returns U.
+// Work in t = a+ - u (Psi decreases in t) with the gap g(t) = log w - log Psi
+// (lower half of w) or log(1 - Psi) - log(1 - w) (upper half), increasing in t
+// and >= 0 exactly when Psi(a+ - t) <= w:
+//  1. bracket: NT candidates t_k = s0 2^(k/8 - 8) (the paper's doubling of the
+//     bracket, eight steps per octave, all at once), s0 = 1/max(1, |a-|) the
+//     scale of the residual's spread;
+//  2. two rounds of NT-way multisection;
+//  3. a secant step between the bracket ends (g known there).
+template <int NT>
+__device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits,
+                                               uint32_t* status, USampleScratch* sm) {
   const unsigned FULL = 0xffffffffu;
-  const int lane = threadIdx.x & 31;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const UParams P = usample_setup(D, la);
   const bool upper = wbits >= 0x80000000u;
   const float target = upper ? logf(((float)(0xFFFFFFFFu - wbits) + 0.5f) * 0x1p-32f)
                              : logf(((float)wbits + 0.5f) * 0x1p-32f);
-  auto below_w = [&](float t) -> bool {  // Psi(a+ - t) <= w
-    if (upper) return usample_log_1mpsi(t, P) >= target;
-    return usample_log_psi(t, P) <= target;
+  auto gap = [&](float t) -> float {
+    if (upper) return usample_log_1mpsi(t, P) - target;
+    return target - usample_log_psi(t, P);
   };
-  float tk = ldexpf(1.0f, lane - 12);
-  unsigned m = __ballot_sync(FULL, below_w(tk));
-  if (m == 0u) {
+  auto first_true = [&](bool pred) -> int {  // smallest tid with pred (NT if none)
+    const unsigned m = __ballot_sync(FULL, pred);
+    if (lane == 0) sm->first[warp] = m ? warp * 32 + __ffs(m) - 1 : NT;
+    __syncthreads();
+    int f = NT;
+#pragma unroll
+    for (int w = 0; w < NT / 32; ++w) f = min(f, sm->first[w]);
+    __syncthreads();
+    return f;
+  };
+  const float s0 = 1.0f / fmaxf(1.0f, fabsf(P.am));
+  const float tk = s0 * exp2f((float)tid * 0.125f - 8.0f);
+  const float gk = gap(tk);
+  int f = first_true(gk >= 0.0f);
+  if (f == NT) {
     *status |= 4u;  // SDV_STATUS_USAMPLE_RANGE
-    return P.ap - ldexpf(1.0f, 19);
+    return P.ap - s0 * exp2f((float)NT * 0.125f - 8.0f);
   }
-  int f = __ffs(m) - 1;
-  float hi = __shfl_sync(FULL, tk, f);
-  float lo = (f == 0) ? 0.0f : __shfl_sync(FULL, tk, f - 1 < 0 ? 0 : f - 1);
+  if (tid == f) { sm->t[1] = tk; sm->g[1] = gk; }
+  if (tid == f - 1) { sm->t[0] = tk; sm->g[0] = gk; }
+  __syncthreads();
+  float hi = sm->t[1], ghi = sm->g[1];
+  float lo = (f == 0) ? 0.0f : sm->t[0];
+  float glo = (f == 0) ? -INFINITY : sm->g[0];
+  __syncthreads();
 #pragma unroll 1
-  for (int round = 0; round < 5; ++round) {
-    const float h = (hi - lo) * (1.0f / 32.0f);
-    const float t = (lane < 31) ? lo + (float)(lane + 1) * h : hi;
-    const bool c = (lane < 31) ? below_w(t) : true;
-    m = __ballot_sync(FULL, c);
-    f = __ffs(m) - 1;
-    const float nhi = __shfl_sync(FULL, t, f);
-    const float nlo = __shfl_sync(FULL, t, f > 0 ? f - 1 : 0);
-    lo = (f == 0) ? lo : nlo;
-    hi = nhi;
+  for (int round = 0; round < 2; ++round) {
+    const float h = (hi - lo) * (1.0f / (float)NT);
+    const float t = (tid < NT - 1) ? lo + (float)(tid + 1) * h : hi;
+    const float gt = (tid < NT - 1) ? gap(t) : ghi;
+    f = first_true(gt >= 0.0f);
+    if (tid == f) { sm->t[1] = t; sm->g[1] = gt; }
+    if (tid == f - 1) { sm->t[0] = t; sm->g[0] = gt; }
+    __syncthreads();
+    if (f > 0) { lo = sm->t[0]; glo = sm->g[0]; }
+    hi = sm->t[1];
+    ghi = sm->g[1];
+    __syncthreads();
   }
-  return P.ap - 0.5f * (lo + hi);
+  float t;
+  if (isfinite(glo) && isfinite(ghi) && ghi > glo) {
+    const float frac = fminf(fmaxf(-glo / (ghi - glo), 0.0f), 1.0f);
+    t = lo + frac * (hi - lo);
+  } else {
+    t = 0.5f * (lo + hi);
+  }
+  return P.ap - t;
 }
 
 // ---------------------------------------------------------------- element access

@@ -8,14 +8,17 @@
 
 namespace sdv {
 
-// K1: threads per CTA and 16-byte vectors per thread per tensor per sweep.
+// Fused verify kernel: threads per CTA and 16-byte vectors per thread per tensor per sweep.
 constexpr int kK1Threads = 256;
 constexpr int kK1Vpt = 4;
-// K2: one warp per chain.
+// Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;
-// K4: threads per CTA and elements of the rejected row per CTA.
+// Long-row residual kernels: threads per CTA and elements of the rejected row per CTA.
 constexpr int kK4Threads = 256;
 constexpr int kK4Chunk = 4096;
+// Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
+// finishes the chain inside the fused kernel; longer rows by k_resid_dot/_write.
+constexpr int64_t kFusedMaxGroups = 4096;
 
 enum : int32_t {
   kKindInactive = 0,
@@ -26,18 +29,19 @@ enum : int32_t {
   kKindBonus = 5,      // full accept, bonus step
 };
 
-// Per-chain result of K2, consumed by K4 (32 bytes).
+// Per-chain result of the scan, consumed by the residual writer (48 bytes).
 struct ChainState {
   int32_t tau;      // 1-based
-  int32_t row;      // row of the window K4 reads (tau-1, or the last draft)
+  int32_t row;      // row of the window the residual writer reads (tau-1, or the last draft)
   float U;          // residual 1-D draw
   float la_res;     // log alpha_{tau-1}
   float sigma;      // sigma_tau
+  float dnorm;      // |Delta_tau|
   float inv_norm;   // 1/|delta_tau|, delta = m^p - m^q
   float refl;       // 1 + 2 S1/S2 (reflection: y = x - delta * refl)
   uint32_t status;
   int32_t kind;
-  int32_t pad;
+  int32_t pad[2];
 };
 
 struct ScanArgs {
@@ -62,7 +66,7 @@ struct ScanArgs {
   float* la_res_out;
   uint32_t* status_out;
   float* aux_out;
-  ChainState* state;
+  bool draw_u;  // draw the residual U (the whole verify step) or stop at tau
 };
 
 struct WsLayout {
@@ -70,7 +74,7 @@ struct WsLayout {
   int64_t chunk1;  // elements of a row per K1 tile
   int C1;          // K1 tiles per row
   int C4;          // K4 tiles per chain
-  size_t part_off, state_off, part4_off, total;
+  size_t ticket_off, part_off, state_off, part4_off, total;
 };
 
 WsLayout ws_layout(int B, int L, int64_t d, int dtype);

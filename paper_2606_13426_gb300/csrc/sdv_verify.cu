@@ -1,24 +1,28 @@
 // sdv_verify.cu - verification step of speculative diffusion sampling on sm_103a.
 //
-// Kernels of one sdv_verify call (all launched on the caller's stream):
-//   K1 ratio_partials : streams x, m^q, m^p once (16-byte loads) and reduces, per
-//                       (chain, step, d-chunk), S1 = sum (x - m^p)(m^p - m^q) and
-//                       S2 = sum (m^p - m^q)^2 (App. "Density ratio calculations":
-//                       Z^T Delta = S1/sigma^2, |Delta|^2 = S2/sigma^2).
-//   K2 scan           : one warp per chain: ell_j, |Delta_j|, the coins, sample or
-//                       block acceptance (Algorithms token-/block-verification), and
-//                       the residual draw U (Algorithm u-sample, warp multisection).
-//   K4a resid_dot     : sum_i delta_i G_i over the rejected row (e^T G up to 1/|delta|).
-//   K4b resid_write   : y = m^q + sigma (U e + G - e e^T G) (Algorithm decomposition-res),
-//                       or the reflection (Algorithm reflect-res), the bonus step,
-//                       or the last accepted draft.
+// One sdv_verify call launches (on the caller's stream) a counter reset and ONE
+// fused kernel, k_verify:
+//   * every CTA streams one tile (chain b, step j, chunk c) of x, m^q and m^p once
+//     with 16-byte loads and reduces S1 = sum (x - m^p)(m^p - m^q) and
+//     S2 = sum (m^p - m^q)^2 (App. "Density ratio calculations": Z^T Delta =
+//     S1/sigma^2, |Delta|^2 = S2/sigma^2), then takes a ticket on its chain;
+//   * the CTA holding a chain's last ticket finishes that chain: warp 0 forms
+//     ell_j and |Delta_j|, draws the coins, applies sample or block acceptance
+//     (Algorithms token-/block-verification) and draws U (Algorithm u-sample);
+//     then the whole CTA writes y (Algorithm decomposition-res: y = m^q +
+//     sigma (U e + G - e e^T G); or reflect-res, the bonus step, or the last
+//     accepted draft).
+// Chains finish at staggered times, so the latency-bound per-chain work overlaps
+// the streaming of other chains.  Rows longer than kFusedMaxGroups groups of four
+// elements are written by two extra kernels (k_resid_dot, k_resid_write) spread
+// over many CTAs.
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
-#include <algorithm>
 #include <vector>
 
 #include "sdv_device.cuh"
@@ -26,10 +30,9 @@
 
 namespace sdv {
 
-// ---------------------------------------------------------------- block reduce
+// ---------------------------------------------------------------- small helpers
 template <int NT>
-__device__ __forceinline__ float2 block_sum2(float a, float b) {
-  __shared__ float2 red[NT / 32];
+__device__ __forceinline__ float2 block_sum2(float a, float b, float2* red) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     a += __shfl_xor_sync(0xffffffffu, a, o);
@@ -50,7 +53,6 @@ __device__ __forceinline__ float2 block_sum2(float a, float b) {
   return r;  // valid in thread 0
 }
 
-// ---------------------------------------------------------------- 16-byte vectors
 __device__ __forceinline__ void unpack(const uint4& v, float (&f)[4]) {
   f[0] = __uint_as_float(v.x);
   f[1] = __uint_as_float(v.y);
@@ -66,286 +68,15 @@ __device__ __forceinline__ void unpack(const uint4& v, float (&f)[8]) {
   }
 }
 
+// Read-once streaming load: no L1 allocation.
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   uint4 r;
   asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
-               : "l"(p));
+      : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+      : "l"(p));
   return r;
 }
 
-// ---------------------------------------------------------------- K1
-template <typename T, bool VEC, int VPT>
-__global__ void __launch_bounds__(kK1Threads)
-k_ratio_partials(const T* __restrict__ x, const T* __restrict__ mq, const T* __restrict__ mp,
-                 int L, int64_t d, int C, int64_t chunk, const int32_t* __restrict__ L_eff,
-                 float2* __restrict__ part) {
-  const int64_t tile = blockIdx.x;
-  const int64_t r = tile / C;
-  const int c = (int)(tile - r * C);
-  const int b = (int)(r / L), j = (int)(r - (int64_t)b * L);
-  if (L_eff != nullptr && j >= L_eff[b]) return;
-  const int64_t e0 = (int64_t)c * chunk;
-  const int64_t e1 = min(e0 + chunk, d);
-  const int64_t base = r * d;
-  float s1 = 0.f, s2 = 0.f;
-  if (VEC) {
-    constexpr int V = 16 / (int)sizeof(T);
-    const int64_t v0 = (base + e0) / V;
-    const int nv = (int)((e1 - e0) / V);
-    const uint4* X = reinterpret_cast<const uint4*>(x) + v0;
-    const uint4* Q = reinterpret_cast<const uint4*>(mq) + v0;
-    const uint4* P = reinterpret_cast<const uint4*>(mp) + v0;
-#pragma unroll 1
-    for (int v = threadIdx.x; v < nv; v += kK1Threads * VPT) {
-      uint4 bx[VPT], bq[VPT], bp[VPT];
-      if (v + (VPT - 1) * kK1Threads < nv) {
-        // full sweep: issue all 3 * VPT 16-byte loads before any use
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) bx[u] = ldg_stream(X + v + u * kK1Threads);
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) bq[u] = ldg_stream(Q + v + u * kK1Threads);
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) bp[u] = ldg_stream(P + v + u * kK1Threads);
-      } else {
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) {
-          const int vv = v + u * kK1Threads;
-          const bool ok = vv < nv;
-          bx[u] = ok ? ldg_stream(X + vv) : make_uint4(0u, 0u, 0u, 0u);
-          bq[u] = ok ? ldg_stream(Q + vv) : make_uint4(0u, 0u, 0u, 0u);
-          bp[u] = ok ? ldg_stream(P + vv) : make_uint4(0u, 0u, 0u, 0u);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < VPT; ++u) {
-        float fx[V], fq[V], fp[V];
-        unpack(bx[u], fx);
-        unpack(bq[u], fq);
-        unpack(bp[u], fp);
-#pragma unroll
-        for (int k = 0; k < V; ++k) {
-          const float dl = fp[k] - fq[k];   // m^p - m^q
-          const float a = fx[k] - fp[k];    // yhat - m^p
-          s1 = fmaf(a, dl, s1);
-          s2 = fmaf(dl, dl, s2);
-        }
-      }
-    }
-  } else {
-    for (int64_t e = e0 + threadIdx.x; e < e1; e += kK1Threads) {
-      const float fx = Elem<T>::load(x + base + e);
-      const float fq = Elem<T>::load(mq + base + e);
-      const float fp = Elem<T>::load(mp + base + e);
-      const float dl = fp - fq, a = fx - fp;
-      s1 = fmaf(a, dl, s1);
-      s2 = fmaf(dl, dl, s2);
-    }
-  }
-  const float2 t = block_sum2<kK1Threads>(s1, s2);
-  if (threadIdx.x == 0) part[tile] = t;
-}
-
-// ---------------------------------------------------------------- K2
-__device__ __forceinline__ float warp_incl_sum(float v, int lane) {
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float t = __shfl_up_sync(0xffffffffu, v, o);
-    if (lane >= o) v += t;
-  }
-  return v;
-}
-__device__ __forceinline__ float warp_incl_max(float v, int lane) {
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const float t = __shfl_up_sync(0xffffffffu, v, o);
-    if (lane >= o) v = fmaxf(v, t);
-  }
-  return v;
-}
-
-__global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
-  const unsigned FULL = 0xffffffffu;
-  const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * (kK2Threads / 32) + (threadIdx.x >> 5);
-  if (b >= A.B) return;  // warp-uniform
-  const int L = A.L;
-  // window length gamma_k, clamped to [0, L] (device data the host cannot check)
-  const int g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
-  if (g <= 0) {
-    if (lane == 0) {
-      if (A.accepted_len) A.accepted_len[b] = 0;
-      if (A.tau_out) A.tau_out[b] = 0;
-      if (A.state) A.state[b] = ChainState{0, -1, NAN, 0.f, 0.f, 0.f, 0.f, 0u, kKindInactive, 0};
-    }
-    if (A.ell_out)
-      for (int j = lane; j < L; j += 32) A.ell_out[(int64_t)b * L + j] = 0.f;
-    if (A.dn_out)
-      for (int j = lane; j < L; j += 32) A.dn_out[(int64_t)b * L + j] = 0.f;
-    return;
-  }
-  const int nseg = (L + 31) >> 5;
-  float ell[2], dn[2], S1[2], S2[2], sg[2];
-  bool bad = false;
-#pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    const int j = lane + 32 * q;
-    ell[q] = 0.f; dn[q] = 0.f; S1[q] = 0.f; S2[q] = 0.f; sg[q] = 1.f;
-    if (q < nseg && j < g) {
-      if (A.part) {
-        const float2* p = A.part + ((int64_t)b * L + j) * A.C;
-        float a1 = 0.f, a2 = 0.f;
-        for (int c = 0; c < A.C; ++c) {
-          const float2 t = p[c];
-          a1 += t.x;
-          a2 += t.y;
-        }
-        const float s = A.sigma[(int64_t)b * A.sstride + j];
-        S1[q] = a1; S2[q] = a2; sg[q] = s;
-        ell[q] = -(a1 + 0.5f * a2) / (s * s);
-        dn[q] = sqrtf(a2) / s;
-        if (!(s > 0.f) || !isfinite(s)) bad = true;
-      } else {
-        ell[q] = A.ell_in[(int64_t)b * L + j];
-        dn[q] = A.dn_in[(int64_t)b * L + j];
-      }
-      if (!isfinite(ell[q]) || !isfinite(dn[q])) bad = true;
-    }
-    if (q < nseg && j < L) {
-      if (A.ell_out) A.ell_out[(int64_t)b * L + j] = ell[q];
-      if (A.dn_out) A.dn_out[(int64_t)b * L + j] = dn[q];
-    }
-  }
-  const bool any_bad = __any_sync(FULL, bad);
-  if (A.ratios_only) return;
-
-  // coins: eta_j from Philox (b, j, 0, 0), word 0, compared in log space
-  float leta[2];
-#pragma unroll
-  for (int q = 0; q < 2; ++q) {
-    const int j = lane + 32 * q;
-    leta[q] = 0.f;
-    if (q < nseg && j < g)
-      leta[q] = log_uniform(philox_block(A.seed, (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
-  }
-  float ellw[2] = {ell[0] * A.inv_omega2, ell[1] * A.inv_omega2};
-
-  int tau;            // 1-based
-  float la_res = 0.f; // log alpha_{tau-1}
-  if (A.mode == 0) {
-    // sample verification: c_j = [eta_j < min{1, e^ell_j}]; tau = first failure
-    unsigned fm[2];
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int j = lane + 32 * q;
-      const bool fail = (q < nseg && j < g) && !(leta[q] < fminf(0.f, ellw[q]));
-      fm[q] = __ballot_sync(FULL, fail);
-    }
-    tau = fm[0] ? __ffs(fm[0]) : (fm[1] ? 32 + __ffs(fm[1]) : g + 1);
-  } else {
-    // block verification: log alpha_j = P_j - max(0, max_{m<=j} P_m), P = prefix sums of ell
-    float la[2];
-    float carryP = 0.f, carryM = 0.f;
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int j = lane + 32 * q;
-      const float v = (q < nseg && j < g) ? ellw[q] : 0.f;
-      float P = warp_incl_sum(v, lane) + carryP;
-      float M = fmaxf(warp_incl_max(P, lane), carryM);
-      M = fmaxf(M, 0.f);
-      la[q] = fminf(P - M, 0.f);
-      carryP = __shfl_sync(FULL, P, 31);
-      carryM = __shfl_sync(FULL, M, 31);
-    }
-    // h_j (0-based j): uses |Delta_{j+2}| in paper numbering = dn at j+1
-    const float dn_next0 = __shfl_down_sync(FULL, dn[0], 1);
-    const float dn_first1 = __shfl_sync(FULL, dn[1], 0);
-    const float dn_next1 = __shfl_down_sync(FULL, dn[1], 1);
-    unsigned sm[2];
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int j = lane + 32 * q;
-      bool succ = false;
-      if (q < nseg && j < g) {
-        float lh;
-        if (j == g - 1) {
-          lh = la[q];                                     // h_gamma = alpha_gamma
-        } else {
-          const float Dn = (q == 0) ? (lane == 31 ? dn_first1 : dn_next0) : dn_next1;
-          lh = block_log_h(la[q], Dn);
-        }
-        succ = leta[q] < lh;
-      }
-      sm[q] = __ballot_sync(FULL, succ);
-    }
-    int last = -1;  // 0-based index of the last success
-    if (sm[1]) last = 32 + 31 - __clz(sm[1]);
-    else if (sm[0]) last = 31 - __clz(sm[0]);
-    tau = last + 2;
-    if (tau >= 2) {
-      const int k = tau - 2;
-      const float v0 = __shfl_sync(FULL, la[0], k & 31);
-      const float v1 = __shfl_sync(FULL, la[1], k & 31);
-      la_res = (k < 32) ? v0 : v1;
-    }
-  }
-
-  // quantities of step tau (0-based row tau-1) when a residual is drawn
-  const bool resid = tau <= g;
-  const int rrow = resid ? tau - 1 : 0;
-  const int rq = rrow >> 5, rl = rrow & 31;
-  const float Dt = rq ? __shfl_sync(FULL, dn[1], rl) : __shfl_sync(FULL, dn[0], rl);
-  const float st = rq ? __shfl_sync(FULL, sg[1], rl) : __shfl_sync(FULL, sg[0], rl);
-  const float S1t = rq ? __shfl_sync(FULL, S1[1], rl) : __shfl_sync(FULL, S1[0], rl);
-  const float S2t = rq ? __shfl_sync(FULL, S2[1], rl) : __shfl_sync(FULL, S2[0], rl);
-
-  uint32_t status = any_bad ? 2u : 0u;
-  float U = NAN;
-  int kind;
-  if (!resid) {
-    kind = A.has_bonus ? kKindBonus : kKindCopy;
-  } else if (!(S2t > 0.f) || !(Dt > 0.f)) {
-    kind = kKindZeroDelta;
-    status |= 1u;
-  } else if (A.residual_kind == 1) {
-    kind = kKindReflect;
-  } else {
-    kind = kKindResid;
-    if (A.state) {
-      const uint32_t wbits = philox_block(A.seed, (uint32_t)b, 0u, kStreamUSample, 0u).x;
-      U = usample_warp(Dt, fminf(la_res, 0.f), wbits, &status);
-    }
-  }
-  if (lane == 0) {
-    if (A.accepted_len) A.accepted_len[b] = tau - 1;
-    if (A.tau_out) A.tau_out[b] = tau;
-    if (A.la_res_out) A.la_res_out[b] = la_res;
-    if (A.status_out) A.status_out[b] = status;
-    if (A.aux_out) {
-      float* a = A.aux_out + 4 * (int64_t)b;
-      a[0] = U;
-      a[1] = la_res;
-      a[2] = resid ? Dt : NAN;
-      a[3] = resid ? st : NAN;
-    }
-    if (A.state) {
-      ChainState cs;
-      cs.tau = tau;
-      cs.row = resid ? rrow : g - 1;
-      cs.U = U;
-      cs.la_res = la_res;
-      cs.sigma = st;
-      cs.inv_norm = (S2t > 0.f) ? rsqrtf(S2t) : 0.f;
-      cs.refl = (S2t > 0.f) ? 1.0f + 2.0f * S1t / S2t : 0.f;
-      cs.status = status;
-      cs.kind = kind;
-      cs.pad = 0;
-      A.state[b] = cs;
-    }
-  }
-}
-
-// ---------------------------------------------------------------- K4a / K4b
 template <typename T, bool VEC4>
 __device__ __forceinline__ void load4(const T* p, int64_t i, int64_t d, float (&f)[4]) {
   if (VEC4 && i + 4 <= d) {
@@ -383,10 +114,439 @@ __device__ __forceinline__ void store4(T* p, int64_t i, int64_t d, const float (
   }
 }
 
+// ---------------------------------------------------------------- tile reduction
+// (S1, S2) of elements [e0, e1) of the row starting at element `base`;
+// VEC: whole 16-byte vectors, VPT of them per thread and tensor per sweep.
+template <typename T, bool VEC, int VPT>
+__device__ __forceinline__ float2 tile_sums(const T* __restrict__ x, const T* __restrict__ mq,
+                                            const T* __restrict__ mp, int64_t base, int64_t e0,
+                                            int64_t e1) {
+  float s1 = 0.f, s2 = 0.f;
+  if (VEC) {
+    constexpr int V = 16 / (int)sizeof(T);
+    const int64_t v0 = (base + e0) / V;
+    const int nv = (int)((e1 - e0) / V);
+    const uint4* X = reinterpret_cast<const uint4*>(x) + v0;
+    const uint4* Q = reinterpret_cast<const uint4*>(mq) + v0;
+    const uint4* P = reinterpret_cast<const uint4*>(mp) + v0;
+#pragma unroll 1
+    for (int v = threadIdx.x; v < nv; v += kK1Threads * VPT) {
+      uint4 bx[VPT], bq[VPT], bp[VPT];
+      if (v + (VPT - 1) * kK1Threads < nv) {
+        // full sweep: issue all 3 * VPT 16-byte loads before any use
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bx[u] = ldg_stream(X + v + u * kK1Threads);
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bq[u] = ldg_stream(Q + v + u * kK1Threads);
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) bp[u] = ldg_stream(P + v + u * kK1Threads);
+      } else {
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) {
+          const int vv = v + u * kK1Threads;
+          const bool ok = vv < nv;
+          bx[u] = ok ? ldg_stream(X + vv) : make_uint4(0u, 0u, 0u, 0u);
+          bq[u] = ok ? ldg_stream(Q + vv) : make_uint4(0u, 0u, 0u, 0u);
+          bp[u] = ok ? ldg_stream(P + vv) : make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < VPT; ++u) {
+        float fx[V], fq[V], fp[V];
+        unpack(bx[u], fx);
+        unpack(bq[u], fq);
+        unpack(bp[u], fp);
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+          const float dl = fp[k] - fq[k];  // m^p - m^q
+          const float a = fx[k] - fp[k];   // yhat - m^p
+          s1 = fmaf(a, dl, s1);
+          s2 = fmaf(dl, dl, s2);
+        }
+      }
+    }
+  } else {
+    for (int64_t e = e0 + threadIdx.x; e < e1; e += kK1Threads) {
+      const float fx = Elem<T>::load(x + base + e);
+      const float fq = Elem<T>::load(mq + base + e);
+      const float fp = Elem<T>::load(mp + base + e);
+      const float dl = fp - fq, a = fx - fp;
+      s1 = fmaf(a, dl, s1);
+      s2 = fmaf(dl, dl, s2);
+    }
+  }
+  return make_float2(s1, s2);
+}
+
+// ---------------------------------------------------------------- chain scan (one warp)
+__device__ __forceinline__ ChainState inactive_state() {
+  ChainState cs;
+  cs.tau = 0; cs.row = -1; cs.U = NAN; cs.la_res = 0.f; cs.sigma = NAN; cs.dnorm = NAN;
+  cs.inv_norm = 0.f; cs.refl = 0.f; cs.status = 0u; cs.kind = kKindInactive;
+  cs.pad[0] = cs.pad[1] = 0;
+  return cs;
+}
+
+// For chain b: ell_j, |Delta_j| (from the tile partials, or given), coins, the
+// acceptance rule, and the residual 1-D draw.  Called by a full warp; every lane
+// returns the chain's ChainState.  Writes the per-chain outputs of ScanArgs.
+__device__ ChainState scan_warp(const ScanArgs& A, int b) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int L = A.L;
+  // window length gamma_k, clamped to [0, L] (device data the host cannot check)
+  const int g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
+  if (g <= 0) {
+    if (lane == 0) {
+      if (A.accepted_len) A.accepted_len[b] = 0;
+      if (A.tau_out) A.tau_out[b] = 0;
+    }
+    if (A.ell_out)
+      for (int j = lane; j < L; j += 32) A.ell_out[(int64_t)b * L + j] = 0.f;
+    if (A.dn_out)
+      for (int j = lane; j < L; j += 32) A.dn_out[(int64_t)b * L + j] = 0.f;
+    return inactive_state();
+  }
+  const int nseg = (L + 31) >> 5;
+  float ell[2], dn[2], S1[2], S2[2], sg[2];
+  bool bad = false;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int j = lane + 32 * q;
+    ell[q] = 0.f; dn[q] = 0.f; S1[q] = 0.f; S2[q] = 0.f; sg[q] = 1.f;
+    if (q < nseg && j < g) {
+      if (A.part) {
+        // partials written by other CTAs of this grid: read through L2
+        const float2* p = A.part + ((int64_t)b * L + j) * A.C;
+        float a1 = 0.f, a2 = 0.f;
+        for (int c = 0; c < A.C; ++c) {
+          const float2 t = __ldcg(p + c);
+          a1 += t.x;
+          a2 += t.y;
+        }
+        const float s = A.sigma[(int64_t)b * A.sstride + j];
+        S1[q] = a1; S2[q] = a2; sg[q] = s;
+        ell[q] = -(a1 + 0.5f * a2) / (s * s);
+        dn[q] = sqrtf(a2) / s;
+        if (!(s > 0.f) || !isfinite(s)) bad = true;
+      } else {
+        ell[q] = A.ell_in[(int64_t)b * L + j];
+        dn[q] = A.dn_in[(int64_t)b * L + j];
+      }
+      if (!isfinite(ell[q]) || !isfinite(dn[q])) bad = true;
+    }
+    if (q < nseg && j < L) {
+      if (A.ell_out) A.ell_out[(int64_t)b * L + j] = ell[q];
+      if (A.dn_out) A.dn_out[(int64_t)b * L + j] = dn[q];
+    }
+  }
+  const bool any_bad = __any_sync(FULL, bad);
+  if (A.ratios_only) return inactive_state();
+
+  // coins: eta_j from Philox (b, j, 0, 0), word 0, compared in log space
+  float leta[2];
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int j = lane + 32 * q;
+    leta[q] = 0.f;
+    if (q < nseg && j < g)
+      leta[q] = log_uniform(philox_block(A.seed, (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
+  }
+  const float ellw[2] = {ell[0] * A.inv_omega2, ell[1] * A.inv_omega2};
+
+  int tau;             // 1-based
+  float la_res = 0.f;  // log alpha_{tau-1}
+  if (A.mode == 0) {
+    // sample verification: c_j = [eta_j < min{1, e^ell_j}]; tau = first failure
+    unsigned fm[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int j = lane + 32 * q;
+      const bool fail = (q < nseg && j < g) && !(leta[q] < fminf(0.f, ellw[q]));
+      fm[q] = __ballot_sync(FULL, fail);
+    }
+    tau = fm[0] ? __ffs(fm[0]) : (fm[1] ? 32 + __ffs(fm[1]) : g + 1);
+  } else {
+    // block verification: log alpha_j = min{0, log alpha_{j-1} + ell_j}, evaluated in
+    // step order (lane j & 31 of segment j >> 5 keeps log alpha_j), so that a clamp to
+    // alpha = 1 is exact exactly when the recursion reaches it
+    float la[2] = {0.f, 0.f};
+    float run = 0.f;
+#pragma unroll 4
+    for (int j = 0; j < g; ++j) {
+      const float e0 = __shfl_sync(FULL, ellw[0], j & 31);
+      const float e1 = __shfl_sync(FULL, ellw[1], j & 31);
+      run = fminf(0.f, run + (j < 32 ? e0 : e1));
+      if (lane == (j & 31)) {
+        if (j < 32) la[0] = run;
+        else la[1] = run;
+      }
+    }
+    // h_j (0-based j) uses |Delta| of step j + 1 (the paper's D_{j+1} in 1-based steps)
+    const float dn_next0 = __shfl_down_sync(FULL, dn[0], 1);
+    const float dn_first1 = __shfl_sync(FULL, dn[1], 0);
+    const float dn_next1 = __shfl_down_sync(FULL, dn[1], 1);
+    unsigned sm[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int j = lane + 32 * q;
+      bool succ = false;
+      if (q < nseg && j < g) {
+        float lh;
+        if (j == g - 1) {
+          lh = la[q];  // h_gamma = alpha_gamma
+        } else {
+          const float Dn = (q == 0) ? (lane == 31 ? dn_first1 : dn_next0) : dn_next1;
+          lh = block_log_h(la[q], Dn);
+        }
+        succ = leta[q] < lh;
+      }
+      sm[q] = __ballot_sync(FULL, succ);
+    }
+    int last = -1;  // 0-based index of the last success
+    if (sm[1]) last = 32 + 31 - __clz(sm[1]);
+    else if (sm[0]) last = 31 - __clz(sm[0]);
+    tau = last + 2;
+    if (tau >= 2) {
+      const int k = tau - 2;
+      const float v0 = __shfl_sync(FULL, la[0], k & 31);
+      const float v1 = __shfl_sync(FULL, la[1], k & 31);
+      la_res = (k < 32) ? v0 : v1;
+    }
+  }
+
+  // quantities of step tau (0-based row tau-1) when a residual is drawn
+  const bool resid = tau <= g;
+  const int rrow = resid ? tau - 1 : 0;
+  const int rq = rrow >> 5, rl = rrow & 31;
+  const float Dt = rq ? __shfl_sync(FULL, dn[1], rl) : __shfl_sync(FULL, dn[0], rl);
+  const float st = rq ? __shfl_sync(FULL, sg[1], rl) : __shfl_sync(FULL, sg[0], rl);
+  const float S1t = rq ? __shfl_sync(FULL, S1[1], rl) : __shfl_sync(FULL, S1[0], rl);
+  const float S2t = rq ? __shfl_sync(FULL, S2[1], rl) : __shfl_sync(FULL, S2[0], rl);
+
+  uint32_t status = any_bad ? 2u : 0u;
+  int kind;
+  if (!resid) {
+    kind = A.has_bonus ? kKindBonus : kKindCopy;
+  } else if (!(S2t > 0.f) || !(Dt > 0.f)) {
+    kind = kKindZeroDelta;
+    status |= 1u;
+  } else if (A.residual_kind == 1) {
+    kind = kKindReflect;
+  } else {
+    kind = kKindResid;
+  }
+  if (lane == 0) {
+    if (A.accepted_len) A.accepted_len[b] = tau - 1;
+    if (A.tau_out) A.tau_out[b] = tau;
+    if (A.la_res_out) A.la_res_out[b] = la_res;
+  }
+  ChainState cs;
+  cs.tau = tau;
+  cs.row = resid ? rrow : g - 1;
+  cs.U = NAN;
+  cs.la_res = la_res;
+  cs.sigma = resid ? st : NAN;
+  cs.dnorm = resid ? Dt : NAN;
+  cs.inv_norm = (S2t > 0.f) ? rsqrtf(S2t) : 0.f;
+  cs.refl = (S2t > 0.f) ? 1.0f + 2.0f * S1t / S2t : 0.f;
+  cs.status = status;
+  cs.kind = kind;
+  cs.pad[0] = cs.pad[1] = 0;
+  return cs;
+}
+
+// Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch), then
+// the outputs that depend on it: status bits and (U, log alpha_res, |Delta_tau|, sigma_tau).
+template <int NT>
+__device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, ChainState& cs,
+                                                  USampleScratch* us) {
+  if (cs.kind == kKindResid && A.draw_u) {
+    const uint32_t wbits = philox_block(A.seed, (uint32_t)b, 0u, kStreamUSample, 0u).x;
+    uint32_t st = cs.status;
+    cs.U = usample_block<NT>(cs.dnorm, fminf(cs.la_res, 0.f), wbits, &st, us);
+    cs.status = st;
+  }
+  if (threadIdx.x == 0 && cs.kind != kKindInactive) {
+    if (A.status_out) A.status_out[b] = cs.status;
+    if (A.aux_out) {
+      float* a = A.aux_out + 4 * (int64_t)b;
+      a[0] = cs.U;
+      a[1] = cs.la_res;
+      a[2] = cs.dnorm;
+      a[3] = cs.sigma;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- residual row by one CTA
+// Writes y[b, :] for chain state cs with the whole CTA (blockDim.x threads, a
+// multiple of 32).  Decomposition: pass A reduces delta^T G, pass B writes
+// m^q + sigma (G + e (U - e^T G)), drawing G again (same Philox counters) rather
+// than holding the row on chip.
+template <typename T, bool VEC4>
+__device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
+                             const T* __restrict__ mp, const T* __restrict__ mq_bonus,
+                             const float* __restrict__ sigma_bonus, int L, int64_t d,
+                             uint64_t seed, int b, const ChainState& cs, T* __restrict__ y,
+                             float2* red, float* bcast) {
+  if (cs.kind == kKindInactive) return;
+  const int nt = blockDim.x;
+  const int64_t ng = (d + 3) / 4;
+  const int64_t rbase = ((int64_t)b * L + cs.row) * d;
+  const int64_t ybase = (int64_t)b * d;
+  if (cs.kind == kKindResid) {
+    float sp = 0.f;
+    for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
+      float fq[4], fp[4];
+      load4<T, VEC4>(mq + rbase, 4 * gi, d, fq);
+      load4<T, VEC4>(mp + rbase, 4 * gi, d, fp);
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      sp = fmaf(fp[0] - fq[0], G.x, sp);  // tail lanes load 0 and contribute 0
+      sp = fmaf(fp[1] - fq[1], G.y, sp);
+      sp = fmaf(fp[2] - fq[2], G.z, sp);
+      sp = fmaf(fp[3] - fq[3], G.w, sp);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sp += __shfl_xor_sync(0xffffffffu, sp, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5].x = sp;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      float v = (threadIdx.x < nt / 32) ? red[threadIdx.x].x : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (threadIdx.x == 0) *bcast = cs.U - v * cs.inv_norm;  // U - e^T G
+    }
+    __syncthreads();
+    const float coef = *bcast;
+    for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
+      float fq[4], fp[4], out[4];
+      load4<T, VEC4>(mq + rbase, 4 * gi, d, fq);
+      load4<T, VEC4>(mp + rbase, 4 * gi, d, fp);
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      const float g4[4] = {G.x, G.y, G.z, G.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        out[k] = fq[k] + cs.sigma * fmaf((fp[k] - fq[k]) * cs.inv_norm, coef, g4[k]);
+      store4<T, VEC4>(y + ybase, 4 * gi, d, out);
+    }
+    return;
+  }
+  for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
+    const int64_t i = 4 * gi;
+    float out[4];
+    if (cs.kind == kKindReflect) {
+      float fx[4], fq[4], fp[4];
+      load4<T, VEC4>(x + rbase, i, d, fx);
+      load4<T, VEC4>(mq + rbase, i, d, fq);
+      load4<T, VEC4>(mp + rbase, i, d, fp);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) out[k] = fx[k] - (fp[k] - fq[k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
+    } else if (cs.kind == kKindZeroDelta) {
+      float fq[4];
+      load4<T, VEC4>(mq + rbase, i, d, fq);
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      out[0] = fq[0] + cs.sigma * G.x; out[1] = fq[1] + cs.sigma * G.y;
+      out[2] = fq[2] + cs.sigma * G.z; out[3] = fq[3] + cs.sigma * G.w;
+    } else if (cs.kind == kKindBonus) {
+      float fb[4];
+      load4<T, VEC4>(mq_bonus + ybase, i, d, fb);
+      const float sb = sigma_bonus[b];
+      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamBonus, 0u);
+      out[0] = fb[0] + sb * G.x; out[1] = fb[1] + sb * G.y;
+      out[2] = fb[2] + sb * G.z; out[3] = fb[3] + sb * G.w;
+    } else {  // copy the last accepted draft
+      load4<T, VEC4>(x + rbase, i, d, out);
+    }
+    store4<T, VEC4>(y + ybase, i, d, out);
+  }
+}
+
+// ---------------------------------------------------------------- the fused kernel
+struct VerifyArgs {
+  const void* x;
+  const void* mq;
+  const void* mp;
+  const void* mq_bonus;
+  const float* sigma_bonus;
+  int64_t d;
+  int64_t chunk;
+  void* y;
+  float2* part;          // [B, L, C] tile partials (also read through S.part)
+  unsigned int* ticket;  // [B], zero at launch
+  ChainState* state;     // [B]; written when the residual row is left to k_resid_*
+  ScanArgs S;
+};
+
+// RESID: 1 = this kernel writes y; 0 = it leaves the chain state for k_resid_*.
+template <typename T, bool VEC, int VPT, bool VEC4, int RESID>
+__global__ void __launch_bounds__(kK1Threads, 4) k_verify(VerifyArgs A) {
+  __shared__ float2 red[kK1Threads / 32];
+  __shared__ int last_s;
+  __shared__ float bcast;
+  __shared__ ChainState cs_s;
+  __shared__ USampleScratch us;
+  const int L = A.S.L;
+  const int C = A.S.C;
+  const int64_t tile = blockIdx.x;
+  const int64_t r = tile / C;
+  const int c = (int)(tile - r * C);
+  const int b = (int)(r / L), j = (int)(r - (int64_t)b * L);
+  const int g = A.S.L_eff ? max(0, min(A.S.L_eff[b], L)) : L;
+  const T* x = (const T*)A.x;
+  const T* mq = (const T*)A.mq;
+  const T* mp = (const T*)A.mp;
+  if (g == 0) {
+    // inactive chain: tile (b, 0, 0) writes its outputs, nothing is streamed
+    if (j == 0 && c == 0 && threadIdx.x < 32) {
+      const ChainState cs = scan_warp(A.S, b);
+      if (threadIdx.x == 0 && RESID == 0) A.state[b] = cs;
+    }
+    return;
+  }
+  if (j >= g) return;
+  const int64_t e0 = (int64_t)c * A.chunk;
+  const int64_t e1 = min(e0 + A.chunk, A.d);
+  const float2 s = tile_sums<T, VEC, VPT>(x, mq, mp, r * A.d, e0, e1);
+  const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
+  if (threadIdx.x == 0) {
+    A.part[tile] = t;
+    __threadfence();  // publish the partial before taking the ticket
+    const unsigned int k = atomicAdd(A.ticket + b, 1u);
+    last_s = (k == (unsigned int)(g * C) - 1u);
+  }
+  __syncthreads();
+  if (!last_s) return;
+  __threadfence();  // acquire: every partial of chain b is visible
+  if (threadIdx.x < 32) {
+    const ChainState cs = scan_warp(A.S, b);
+    if (threadIdx.x == 0) cs_s = cs;
+  }
+  __syncthreads();
+  if (A.S.ratios_only) return;
+  ChainState cs = cs_s;
+  draw_u_and_report<kK1Threads>(A.S, b, cs, &us);
+  if (RESID == 0) {
+    if (threadIdx.x == 0) A.state[b] = cs;
+  } else {
+    residual_cta<T, VEC4>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, A.S.seed, b,
+                          cs, (T*)A.y, red, &bcast);
+  }
+}
+
+// ---------------------------------------------------------------- acceptance scan only
+__global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
+  const int b = blockIdx.x * (kK2Threads / 32) + (threadIdx.x >> 5);
+  if (b >= A.B) return;  // warp-uniform
+  scan_warp(A, b);
+}
+
+// ---------------------------------------------------------------- long rows: K4a / K4b
 template <typename T, bool VEC4>
 __global__ void __launch_bounds__(kK4Threads)
 k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d, int C4,
             uint64_t seed, const ChainState* __restrict__ state, float* __restrict__ part4) {
+  __shared__ float2 red[kK4Threads / 32];
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
   const ChainState cs = state[b];
   if (cs.kind != kKindResid) return;
@@ -399,11 +559,12 @@ k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d
     load4<T, VEC4>(mq + base, 4 * gi, d, fq);
     load4<T, VEC4>(mp + base, 4 * gi, d, fp);
     const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-    const float g[4] = {G.x, G.y, G.z, G.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) s = fmaf(fp[k] - fq[k], g[k], s);   // tail lanes load 0
+    s = fmaf(fp[0] - fq[0], G.x, s);
+    s = fmaf(fp[1] - fq[1], G.y, s);
+    s = fmaf(fp[2] - fq[2], G.z, s);
+    s = fmaf(fp[3] - fq[3], G.w, s);
   }
-  const float2 t = block_sum2<kK4Threads>(s, 0.f);
+  const float2 t = block_sum2<kK4Threads>(s, 0.f, red);
   if (threadIdx.x == 0) part4[blockIdx.x] = t.x;
 }
 
@@ -434,19 +595,17 @@ k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __rest
       load4<T, VEC4>(mq + rbase, i, d, fq);
       load4<T, VEC4>(mp + rbase, i, d, fp);
       const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-      const float g[4] = {G.x, G.y, G.z, G.w};
+      const float g4[4] = {G.x, G.y, G.z, G.w};
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const float e = (fp[k] - fq[k]) * cs.inv_norm;
-        out[k] = fq[k] + cs.sigma * fmaf(e, coef, g[k]);   // m^q + sigma (G + e (U - e^T G))
-      }
+      for (int k = 0; k < 4; ++k)
+        out[k] = fq[k] + cs.sigma * fmaf((fp[k] - fq[k]) * cs.inv_norm, coef, g4[k]);
     } else if (cs.kind == kKindReflect) {
       float fx[4], fq[4], fp[4];
       load4<T, VEC4>(x + rbase, i, d, fx);
       load4<T, VEC4>(mq + rbase, i, d, fq);
       load4<T, VEC4>(mp + rbase, i, d, fp);
 #pragma unroll
-      for (int k = 0; k < 4; ++k) out[k] = fx[k] - (fp[k] - fq[k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
+      for (int k = 0; k < 4; ++k) out[k] = fx[k] - (fp[k] - fq[k]) * cs.refl;
     } else if (cs.kind == kKindZeroDelta) {
       float fq[4];
       load4<T, VEC4>(mq + rbase, i, d, fq);
@@ -460,7 +619,7 @@ k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __rest
       const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamBonus, 0u);
       out[0] = fb[0] + sb * G.x; out[1] = fb[1] + sb * G.y;
       out[2] = fb[2] + sb * G.z; out[3] = fb[3] + sb * G.w;
-    } else {  // copy the last accepted draft
+    } else {
       load4<T, VEC4>(x + rbase, i, d, out);
     }
     store4<T, VEC4>(y + ybase, i, d, out);
@@ -468,11 +627,11 @@ k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __rest
 }
 
 // ---------------------------------------------------------------- stand-alone pieces
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(kK1Threads)
 k_usample(const float* __restrict__ D, const float* __restrict__ la, const uint32_t* __restrict__ w,
           int n, float* __restrict__ U, uint32_t* __restrict__ st) {
-  const int i = blockIdx.x * 4 + (threadIdx.x >> 5);
-  if (i >= n) return;  // warp-uniform
+  __shared__ USampleScratch us;
+  const int i = blockIdx.x;  // one CTA per item
   const float Dn = D[i];
   float l = la[i];
   uint32_t status = 0u;
@@ -483,9 +642,9 @@ k_usample(const float* __restrict__ D, const float* __restrict__ la, const uint3
     status = 1u;
   } else {
     l = fminf(l, 0.f);
-    u = usample_warp(Dn, l, w[i], &status);
+    u = usample_block<kK1Threads>(Dn, l, w[i], &status, &us);
   }
-  if ((threadIdx.x & 31) == 0) {
+  if (threadIdx.x == 0) {
     U[i] = u;
     if (st) st[i] = status;
   }
@@ -523,7 +682,7 @@ static int check_launch() {
 static bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // ---- per-thread timing ring (sdv_timing_enable / sdv_timing_read).  Records use
-// cudaEventRecordExternal so that, under stream capture, they become event-record
+// cudaEventRecordExternal under stream capture, so that they become event-record
 // nodes of the graph (a plain record there only expresses a dependency).
 struct TimingRing {
   std::vector<cudaEvent_t> ev;  // slots x 4
@@ -546,6 +705,13 @@ static cudaEvent_t* timing_slot() {
   return &g_timing.ev[4 * (size_t)s];
 }
 
+static void timing_record(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(s, &cap);
+  if (cap == cudaStreamCaptureStatusActive) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+  else cudaEventRecord(e, s);
+}
+
 WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   WsLayout w{};
   const int es = dtype == SDV_BF16 ? 2 : 4;
@@ -558,6 +724,8 @@ WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   w.C4 = (int)((d + kK4Chunk - 1) / kK4Chunk);
   auto up = [](size_t v) { return (v + 255) & ~(size_t)255; };
   size_t off = 0;
+  w.ticket_off = off;
+  off = up(off + sizeof(unsigned int) * (size_t)B);
   w.part_off = off;
   off = up(off + sizeof(float2) * (size_t)B * L * w.C1);
   w.state_off = off;
@@ -581,23 +749,36 @@ static int validate_window(const void* x, const void* mq, const void* mp, const 
   return SDV_OK;
 }
 
-template <typename T>
-static void launch_k1(const void* x, const void* mq, const void* mp, int B, int L, int64_t d,
-                      const int32_t* L_eff, const WsLayout& w, float2* part, cudaStream_t s) {
+template <typename T, int RESID>
+static void launch_verify(const VerifyArgs& A, int B, int L, int vpt, cudaStream_t s) {
   constexpr int V = 16 / (int)sizeof(T);
-  const bool vec = (d % V == 0) && aligned(x, 16) && aligned(mq, 16) && aligned(mp, 16);
-  const unsigned tiles = (unsigned)((int64_t)B * L * w.C1);
-  const T *X = (const T*)x, *Q = (const T*)mq, *P = (const T*)mp;
+  const bool vec = (A.d % V == 0) && aligned(A.x, 16) && aligned(A.mq, 16) && aligned(A.mp, 16);
+  const bool vec4 = (A.d % 4 == 0) && aligned(A.x, 4 * sizeof(T)) && aligned(A.mq, 4 * sizeof(T)) &&
+                    aligned(A.mp, 4 * sizeof(T)) && (A.y == nullptr || aligned(A.y, 4 * sizeof(T))) &&
+                    (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
+  const unsigned tiles = (unsigned)((int64_t)B * L * A.S.C);
+#define SDV_LAUNCH(VECV, VPTV, V4) k_verify<T, VECV, VPTV, V4, RESID><<<tiles, kK1Threads, 0, s>>>(A)
   if (!vec) {
-    k_ratio_partials<T, false, 1><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part);
+    if (vec4) SDV_LAUNCH(false, 1, true);
+    else SDV_LAUNCH(false, 1, false);
     return;
   }
-  switch (w.vpt1) {
-    case 1: k_ratio_partials<T, true, 1><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
-    case 2: k_ratio_partials<T, true, 2><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
-    case 3: k_ratio_partials<T, true, 3><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
-    default: k_ratio_partials<T, true, 4><<<tiles, kK1Threads, 0, s>>>(X, Q, P, L, d, w.C1, w.chunk1, L_eff, part); break;
+  if (vec4) {
+    switch (vpt) {
+      case 1: SDV_LAUNCH(true, 1, true); break;
+      case 2: SDV_LAUNCH(true, 2, true); break;
+      case 3: SDV_LAUNCH(true, 3, true); break;
+      default: SDV_LAUNCH(true, 4, true); break;
+    }
+  } else {
+    switch (vpt) {
+      case 1: SDV_LAUNCH(true, 1, false); break;
+      case 2: SDV_LAUNCH(true, 2, false); break;
+      case 3: SDV_LAUNCH(true, 3, false); break;
+      default: SDV_LAUNCH(true, 4, false); break;
+    }
   }
+#undef SDV_LAUNCH
 }
 
 template <typename T>
@@ -619,13 +800,71 @@ static void launch_k4(const void* x, const void* mq, const void* mp, const void*
   }
 }
 
+// Enqueue the whole step (or, with ratios_only, the log-ratio pass) for validated args.
+static int enqueue_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
+                          const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d,
+                          int dtype, uint64_t seed, int mode, const int32_t* L_eff,
+                          const void* mu_target_bonus, const float* sigma_bonus,
+                          int residual_kind, float omega, int32_t* accepted_len, void* y_out,
+                          float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
+                          float* chain_aux_out, bool ratios_only, void* workspace,
+                          cudaStream_t s) {
+  const WsLayout w = ws_layout(B, L, d, dtype);
+  char* ws = (char*)workspace;
+  VerifyArgs A{};
+  A.x = x_draft; A.mq = mu_target; A.mp = mu_draft;
+  A.mq_bonus = mu_target_bonus; A.sigma_bonus = sigma_bonus;
+  A.d = d; A.chunk = w.chunk1; A.y = y_out;
+  A.ticket = (unsigned int*)(ws + w.ticket_off);
+  A.state = (ChainState*)(ws + w.state_off);
+  ScanArgs& S = A.S;
+  A.part = (float2*)(ws + w.part_off);
+  S.part = A.part; S.C = w.C1; S.sigma = sigma; S.sstride = sigma_stride_b;
+  S.B = B; S.L = L; S.L_eff = L_eff; S.seed = seed; S.mode = mode;
+  S.inv_omega2 = 1.0f / (omega * omega); S.residual_kind = residual_kind;
+  S.has_bonus = mu_target_bonus != nullptr; S.ratios_only = ratios_only; S.draw_u = true;
+  S.ell_out = log_ratio_out; S.dn_out = delta_norm_out; S.accepted_len = accepted_len;
+  S.status_out = status_out; S.aux_out = chain_aux_out;
+
+  cudaEvent_t* tev = ratios_only ? nullptr : timing_slot();
+  if (tev) timing_record(tev[0], s);
+  if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+    check_launch();
+    return SDV_ECUDA;
+  }
+  const bool long_rows = (d + 3) / 4 > kFusedMaxGroups;
+  if (long_rows && !ratios_only) {
+    if (dtype == SDV_F32) launch_verify<float, 0>(A, B, L, w.vpt1, s);
+    else launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, s);
+  } else {
+    if (dtype == SDV_F32) launch_verify<float, 1>(A, B, L, w.vpt1, s);
+    else launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, s);
+  }
+  int rc = check_launch();
+  if (rc != SDV_OK) return rc;
+  if (tev) timing_record(tev[1], s);
+  if (long_rows && !ratios_only) {
+    float* part4 = (float*)(ws + w.part4_off);
+    if (dtype == SDV_F32)
+      launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, A.state, part4, y_out, s);
+    else
+      launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, A.state, part4, y_out, s);
+    rc = check_launch();
+  }
+  if (tev) {
+    timing_record(tev[2], s);
+    timing_record(tev[3], s);
+  }
+  return rc;
+}
+
 }  // namespace sdv
 
 using namespace sdv;
 
 extern "C" {
 
-const char* sdv_version(void) { return "specdiff-gb300 0.1 (sm_103a)"; }
+const char* sdv_version(void) { return "specdiff-gb300 0.2 (sm_103a)"; }
 
 const char* sdv_strerror(int code) {
   switch (code) {
@@ -671,37 +910,85 @@ int sdv_verify_ex(const void* x_draft, const void* mu_target, const void* mu_dra
   const WsLayout w = ws_layout(B, L, d, dtype);
   if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
   if (!aligned(workspace, 256)) return SDV_EALIGN;
-  cudaStream_t s = (cudaStream_t)stream;
-  char* ws = (char*)workspace;
-  float2* part = (float2*)(ws + w.part_off);
-  ChainState* st = (ChainState*)(ws + w.state_off);
-  float* part4 = (float*)(ws + w.part4_off);
+  return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                        mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+                        accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
+                        chain_aux_out, false, workspace, (cudaStream_t)stream);
+}
 
-  cudaEvent_t* tev = timing_slot();
-  if (tev) cudaEventRecordWithFlags(tev[0], s, cudaEventRecordExternal);
-  if (dtype == SDV_F32) launch_k1<float>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
-  else launch_k1<__nv_bfloat16>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
-  if ((rc = check_launch()) != SDV_OK) return rc;
-  if (tev) cudaEventRecordWithFlags(tev[1], s, cudaEventRecordExternal);
+int sdv_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
+               const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+               uint64_t seed, int mode, int32_t* accepted_len, void* y_out,
+               float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
+               void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  return sdv_verify_ex(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                       mode, nullptr, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION, 1.0f,
+                       accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, nullptr,
+                       workspace, workspace_bytes, stream);
+}
 
+int sdv_log_ratios(const void* x_draft, const void* mu_target, const void* mu_draft,
+                   const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                   const int32_t* L_eff, float* log_ratio_out, float* delta_norm_out,
+                   void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
+  if (rc != SDV_OK) return rc;
+  if (!log_ratio_out || !delta_norm_out) return SDV_EINVAL;
+  if (!aligned(log_ratio_out, 4) || !aligned(delta_norm_out, 4) || (L_eff && !aligned(L_eff, 4)))
+    return SDV_EALIGN;
+  const WsLayout w = ws_layout(B, L, d, dtype);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if (!aligned(workspace, 256)) return SDV_EALIGN;
+  return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, 0,
+                        SDV_MODE_BLOCK, L_eff, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION, 1.0f,
+                        nullptr, nullptr, log_ratio_out, delta_norm_out, nullptr, nullptr, true,
+                        workspace, (cudaStream_t)stream);
+}
+
+int sdv_accept_scan(const float* log_ratio, const float* delta_norm, int B, int L,
+                    const int32_t* L_eff, uint64_t seed, int mode, float omega, int32_t* tau_out,
+                    float* log_alpha_res_out, sdv_stream_t stream) {
+  if (!log_ratio || !delta_norm || !tau_out) return SDV_EINVAL;
+  if (B < 1 || L < 1 || L > SDV_MAX_L || B > (1 << 30)) return SDV_EINVAL;
+  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
+  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
+  if (!aligned(log_ratio, 4) || !aligned(delta_norm, 4) || !aligned(tau_out, 4) ||
+      (log_alpha_res_out && !aligned(log_alpha_res_out, 4)) || (L_eff && !aligned(L_eff, 4)))
+    return SDV_EALIGN;
   ScanArgs A{};
-  A.part = part; A.C = w.C1; A.sigma = sigma; A.sstride = sigma_stride_b;
-  A.B = B; A.L = L; A.L_eff = L_eff; A.seed = seed; A.mode = mode;
-  A.inv_omega2 = 1.0f / (omega * omega); A.residual_kind = residual_kind;
-  A.has_bonus = mu_target_bonus != nullptr; A.ratios_only = false;
-  A.ell_out = log_ratio_out; A.dn_out = delta_norm_out; A.accepted_len = accepted_len;
-  A.status_out = status_out; A.aux_out = chain_aux_out; A.state = st;
-  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, s>>>(A);
-  if ((rc = check_launch()) != SDV_OK) return rc;
-  if (tev) cudaEventRecordWithFlags(tev[2], s, cudaEventRecordExternal);
+  A.ell_in = log_ratio; A.dn_in = delta_norm; A.B = B; A.L = L; A.L_eff = L_eff;
+  A.seed = seed; A.mode = mode; A.inv_omega2 = 1.0f / (omega * omega);
+  A.tau_out = tau_out; A.la_res_out = log_alpha_res_out; A.draw_u = false;
+  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, (cudaStream_t)stream>>>(A);
+  return check_launch();
+}
 
-  if (dtype == SDV_F32)
-    launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, st, part4, y_out, s);
-  else
-    launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, st, part4, y_out, s);
-  rc = check_launch();
-  if (tev) cudaEventRecordWithFlags(tev[3], s, cudaEventRecordExternal);
-  return rc;
+int sdv_usample(const float* delta_norm, const float* log_alpha, const uint32_t* w_bits, int n,
+                float* U_out, uint32_t* status_out, sdv_stream_t stream) {
+  if (!delta_norm || !log_alpha || !w_bits || !U_out || n < 0) return SDV_EINVAL;
+  if (!aligned(delta_norm, 4) || !aligned(log_alpha, 4) || !aligned(w_bits, 4) ||
+      !aligned(U_out, 4) || (status_out && !aligned(status_out, 4)))
+    return SDV_EALIGN;
+  if (n == 0) return SDV_OK;
+  k_usample<<<n, kK1Threads, 0, (cudaStream_t)stream>>>(delta_norm, log_alpha, w_bits, n, U_out, status_out);
+  return check_launch();
+}
+
+int sdv_philox(const uint32_t* ctr, uint64_t seed, int n, uint32_t* out, sdv_stream_t stream) {
+  if (!ctr || !out || n < 0) return SDV_EINVAL;
+  if (!aligned(ctr, 16) || !aligned(out, 16)) return SDV_EALIGN;
+  if (n == 0) return SDV_OK;
+  k_philox<<<(n + 255) / 256, 256, 0, (cudaStream_t)stream>>>((const uint4*)ctr, seed, n, (uint4*)out);
+  return check_launch();
+}
+
+int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub, float* out,
+                sdv_stream_t stream) {
+  if (!out || B < 1 || d < 1 || stream_id < 0) return SDV_EINVAL;
+  if (!aligned(out, 4)) return SDV_EALIGN;
+  const int64_t n = (int64_t)B * ((d + 3) / 4);
+  k_normals<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(seed, B, d, (uint32_t)stream_id, sub, out);
+  return check_launch();
 }
 
 int sdv_timing_enable(int slots) {
@@ -743,88 +1030,6 @@ int sdv_timing_read(int n_calls, float* ms3) {
   }
   for (int k = 0; k < 3; ++k) ms3[k] = (float)acc[k];
   return SDV_OK;
-}
-
-int sdv_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
-               const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
-               uint64_t seed, int mode, int32_t* accepted_len, void* y_out,
-               float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
-               void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
-  return sdv_verify_ex(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
-                       mode, nullptr, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION, 1.0f,
-                       accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, nullptr,
-                       workspace, workspace_bytes, stream);
-}
-
-int sdv_log_ratios(const void* x_draft, const void* mu_target, const void* mu_draft,
-                   const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
-                   const int32_t* L_eff, float* log_ratio_out, float* delta_norm_out,
-                   void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
-  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
-  if (rc != SDV_OK) return rc;
-  if (!log_ratio_out || !delta_norm_out) return SDV_EINVAL;
-  if (!aligned(log_ratio_out, 4) || !aligned(delta_norm_out, 4) || (L_eff && !aligned(L_eff, 4)))
-    return SDV_EALIGN;
-  const WsLayout w = ws_layout(B, L, d, dtype);
-  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
-  if (!aligned(workspace, 256)) return SDV_EALIGN;
-  cudaStream_t s = (cudaStream_t)stream;
-  float2* part = (float2*)((char*)workspace + w.part_off);
-  if (dtype == SDV_F32) launch_k1<float>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
-  else launch_k1<__nv_bfloat16>(x_draft, mu_target, mu_draft, B, L, d, L_eff, w, part, s);
-  if ((rc = check_launch()) != SDV_OK) return rc;
-  ScanArgs A{};
-  A.part = part; A.C = w.C1; A.sigma = sigma; A.sstride = sigma_stride_b;
-  A.B = B; A.L = L; A.L_eff = L_eff; A.inv_omega2 = 1.f; A.ratios_only = true;
-  A.ell_out = log_ratio_out; A.dn_out = delta_norm_out;
-  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, s>>>(A);
-  return check_launch();
-}
-
-int sdv_accept_scan(const float* log_ratio, const float* delta_norm, int B, int L,
-                    const int32_t* L_eff, uint64_t seed, int mode, float omega, int32_t* tau_out,
-                    float* log_alpha_res_out, sdv_stream_t stream) {
-  if (!log_ratio || !delta_norm || !tau_out) return SDV_EINVAL;
-  if (B < 1 || L < 1 || L > SDV_MAX_L || B > (1 << 30)) return SDV_EINVAL;
-  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
-  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
-  if (!aligned(log_ratio, 4) || !aligned(delta_norm, 4) || !aligned(tau_out, 4) ||
-      (log_alpha_res_out && !aligned(log_alpha_res_out, 4)) || (L_eff && !aligned(L_eff, 4)))
-    return SDV_EALIGN;
-  ScanArgs A{};
-  A.ell_in = log_ratio; A.dn_in = delta_norm; A.B = B; A.L = L; A.L_eff = L_eff;
-  A.seed = seed; A.mode = mode; A.inv_omega2 = 1.0f / (omega * omega);
-  A.tau_out = tau_out; A.la_res_out = log_alpha_res_out;
-  k_scan<<<(B + kK2Threads / 32 - 1) / (kK2Threads / 32), kK2Threads, 0, (cudaStream_t)stream>>>(A);
-  return check_launch();
-}
-
-int sdv_usample(const float* delta_norm, const float* log_alpha, const uint32_t* w_bits, int n,
-                float* U_out, uint32_t* status_out, sdv_stream_t stream) {
-  if (!delta_norm || !log_alpha || !w_bits || !U_out || n < 0) return SDV_EINVAL;
-  if (!aligned(delta_norm, 4) || !aligned(log_alpha, 4) || !aligned(w_bits, 4) ||
-      !aligned(U_out, 4) || (status_out && !aligned(status_out, 4)))
-    return SDV_EALIGN;
-  if (n == 0) return SDV_OK;
-  k_usample<<<(n + 3) / 4, 128, 0, (cudaStream_t)stream>>>(delta_norm, log_alpha, w_bits, n, U_out, status_out);
-  return check_launch();
-}
-
-int sdv_philox(const uint32_t* ctr, uint64_t seed, int n, uint32_t* out, sdv_stream_t stream) {
-  if (!ctr || !out || n < 0) return SDV_EINVAL;
-  if (!aligned(ctr, 16) || !aligned(out, 16)) return SDV_EALIGN;
-  if (n == 0) return SDV_OK;
-  k_philox<<<(n + 255) / 256, 256, 0, (cudaStream_t)stream>>>((const uint4*)ctr, seed, n, (uint4*)out);
-  return check_launch();
-}
-
-int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub, float* out,
-                sdv_stream_t stream) {
-  if (!out || B < 1 || d < 1 || stream_id < 0) return SDV_EINVAL;
-  if (!aligned(out, 4)) return SDV_EALIGN;
-  const int64_t n = (int64_t)B * ((d + 3) / 4);
-  k_normals<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(seed, B, d, (uint32_t)stream_id, sub, out);
-  return check_launch();
 }
 
 }  // extern "C"

@@ -58,6 +58,16 @@ def near_tie(o, mode, omega=1.0, band=1e-4, rtol=1e-5):
             lh = np.log(o["h"][:, 1:])
         cum = np.cumsum(slack, axis=1)
         tie = np.abs(leta - lh) < band + cum
+        # h_j is discontinuous at alpha_j = 1 when |Delta_{j+1}| = 0 (h = 1 at alpha = 1,
+        # h = 0 for any alpha < 1): a log alpha_j within rounding of 0 there is a tie
+        la = np.zeros((n, L))
+        run = np.zeros(n)
+        for j in range(L):
+            run = np.minimum(0.0, run + ell[:, j])
+            la[:, j] = run
+        dnext = np.concatenate([o["dnorm"][:, 1:], np.ones((n, 1))], axis=1) \
+            if "dnorm" in o else np.ones((n, L))
+        tie |= (dnext == 0.0) & (np.abs(la) < 1e-5 * (1 + np.arange(L)))
     return tie.any(axis=1)
 
 

@@ -128,7 +128,7 @@ def test_accept_scan_matches_oracle(api, mode, m, L):
             to, lao, _, h = OV.block_verification(ell, dn, eta, Leff, omega)
         to = np.where(Leff == 0, 0, to)
         o = dict(ell=ell.astype(np.float64) * np.where(np.arange(L) < Leff[:, None], 1, 0),
-                 eta=eta, h=h)
+                 eta=eta, h=h, dnorm=dn.astype(np.float64))
         from gpu_helpers import near_tie
         diff = tau != to
         assert np.all(near_tie(o, m, omega, rtol=1e-6)[diff]), np.nonzero(diff)[0][:5]
@@ -211,8 +211,10 @@ def test_verify_edge_shapes(api):
         np.testing.assert_array_equal(g["y"], inp["x_draft"][:, -1])
 
 
-def test_zero_delta_residual_is_flagged(api):
-    """Block mode can reject a step whose means coincide: y = m^q + sigma G, status bit 1."""
+def test_zero_delta_step_is_never_the_residual(api):
+    """A step with m^p = m^q is never rejected: in sample mode its ratio is 1, and in block
+    mode h_{j-1} = 0 unless alpha_{j-1} = 1, in which case alpha_j = 1 and h_j = 1.  So the
+    SDV_STATUS_ZERO_DELTA branch (y = m^q + sigma G) is unreachable for exact zeros."""
     rng = np.random.Generator(np.random.PCG64(10))
     Bn, L, d = 4000, 3, 4
     s = np.full((Bn, L), 0.5, np.float32)
@@ -225,12 +227,12 @@ def test_zero_delta_residual_is_flagged(api):
     x = (mp[None] + 0.5 * rng.standard_normal((Bn, L, d))).astype(np.float32)
     inp = dict(x_draft=x, mu_target=np.broadcast_to(mq, x.shape).copy(),
                mu_draft=np.broadcast_to(mp, x.shape).copy(), sigma=s, dtype="f32")
-    g = run_gpu(api, inp, 4, "block")
-    o = oracle_for(inp, 4, OV.MODE_BLOCK)
-    compare(g, o, OV.MODE_BLOCK, "f32")
-    zero = (g["accepted_len"] == 1)
-    assert zero.any()
-    assert np.all(g["status"][zero] & 1)
+    for mode, m in MODES:
+        g = run_gpu(api, inp, 4, mode)
+        o = oracle_for(inp, 4, m)
+        compare(g, o, m, "f32")
+        assert not np.any(g["accepted_len"] == 1)      # tau = 2 would be the zero-delta step
+        assert not np.any(g["status"] & 1)
 
 
 # ------------------------------------------------------------------ statistics on the GPU path

@@ -151,6 +151,36 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
                   void *workspace, size_t workspace_bytes, sdv_stream_t stream);
 
 /*
+ * sdv_verify_noalloc - sdv_verify without a workspace argument, for callers that
+ * cannot allocate device memory.  (The paper has no counterpart; this is a
+ * deployment option of this library.)  Such callers include plug-ins loaded into a
+ * host program that owns every device allocation through its own allocator, and
+ * real-time loops where cudaMalloc's implicit synchronisation and possible failure
+ * are not allowed.  They still pass their inputs and outputs; the scratch comes from
+ * a static device array of SDV_NOALLOC_SCRATCH_BYTES inside this library, which every
+ * GPU that loads the library holds until the process exits.
+ *   - Same arguments, semantics and results as sdv_verify.
+ *   - Returns SDV_ENOWORKSPACE, launching nothing, when
+ *     sdv_workspace_bytes(B, L, d, dtype) > SDV_NOALLOC_SCRATCH_BYTES.
+ *   - Calls no cudaMalloc / cudaFree or any other allocating routine.
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture on the device.
+ *   - Every call on a device shares the one array, which keeps the previous call's
+ *     contents: the counters that must start at zero are cleared by each call on its
+ *     own stream, but calls that overlap on the GPU (other streams, other host
+ *     threads, same device) race on the array.  Serialise them, e.g. on one stream.
+ */
+#define SDV_NOALLOC_SCRATCH_BYTES (1u << 20)
+int sdv_verify_noalloc(const void *x_draft, const void *mu_target, const void *mu_draft,
+                       const float *sigma, int64_t sigma_stride_b,
+                       int B, int L, int64_t d, int dtype,
+                       uint64_t seed, int mode,
+                       int32_t *accepted_len, void *y_out,
+                       float *log_ratio_out, float *delta_norm_out, uint32_t *status_out,
+                       sdv_stream_t stream);
+
+/*
  * sdv_log_ratios - only the fused reduction over d (App. "Density ratio
  * calculations"): ell_j = -Z_j^T Delta_j - |Delta_j|^2/2 and |Delta_j| for
  * every (b, j) with j < L_eff[b] (all j if L_eff is NULL; 0 elsewhere).

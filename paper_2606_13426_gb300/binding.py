@@ -27,6 +27,7 @@ SDV_STATUS_ZERO_DELTA = 1
 SDV_STATUS_NONFINITE = 2
 SDV_STATUS_USAMPLE_RANGE = 4
 SDV_MAX_L = 64
+SDV_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -47,6 +48,8 @@ SIGNATURES = {
     "sdv_verify_ex": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _U64, _I,
                            _P, _P, _P, _I, _F,
                            _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "sdv_verify_noalloc": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _U64, _I,
+                                _P, _P, _P, _P, _P, _P]),
     "sdv_log_ratios": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _P, _P, _P, _P, _SZ, _P]),
     "sdv_accept_scan": (_I, [_P, _P, _I, _I, _P, _U64, _I, _F, _P, _P, _P]),
     "sdv_usample": (_I, [_P, _P, _P, _I, _P, _P, _P]),
@@ -130,6 +133,15 @@ def sdv_verify_ex(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, 
                  dtype, seed, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
                  accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, chain_aux_out,
                  workspace, workspace_bytes, stream)
+
+
+def sdv_verify_noalloc(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                       mode, accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
+                       stream):
+    """sdv_verify with its scratch in the library's static device array (no workspace)."""
+    return _call("sdv_verify_noalloc", x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L,
+                 d, dtype, seed, mode, accepted_len, y_out, log_ratio_out, delta_norm_out,
+                 status_out, stream)
 
 
 def sdv_log_ratios(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, L_eff,

@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIBDIR = os.path.join(PKG, "lib")
 LIBNAME = "libspecdiff.so"
-SOURCES = ["sdv_verify.cu", "sdv_sampler.cu"]
+SOURCES = ["sdv_verify.cu", "sdv_sampler.cu", "sdv_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + INCLUDE,
               "-I" + CSRC]

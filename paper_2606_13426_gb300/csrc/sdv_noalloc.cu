@@ -1,0 +1,70 @@
+// sdv_noalloc.cu - sdv_verify_noalloc: the whole verification step with its
+// scratch memory in a static device array instead of a caller-provided workspace.
+//
+// Who needs this: code that may not call cudaMalloc at all.  Typical cases are
+// plug-ins loaded into a host program that owns every device allocation through
+// its own allocator (custom operators of an inference server, stages of a media
+// or rendering pipeline), and real-time loops where cudaMalloc's implicit device
+// synchronisation and its possible failure at run time are not acceptable.  Such
+// callers can still hand over their input and output buffers; only the scratch
+// has to come from somewhere else.
+//
+// The scratch is a file-scope __device__ array of SDV_NOALLOC_SCRATCH_BYTES.  Every
+// GPU on which this library is loaded holds it until the process exits.  Host code
+// cannot use the array's name as a device address (it is a host-side stand-in), so
+// the device address is fetched with cudaGetSymbolAddress, once per device, with
+// that device current, and passed to the kernels as their workspace.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "sdv_host.h"
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[SDV_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch on the current device (set-up on first use).
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return (int)e;
+  if (dev < 0 || dev >= kMaxDevices) return (int)cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return (int)e;
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return 0;
+}
+
+}  // namespace
+
+extern "C" int sdv_verify_noalloc(const void* x_draft, const void* mu_target, const void* mu_draft,
+                                  const float* sigma, int64_t sigma_stride_b, int B, int L,
+                                  int64_t d, int dtype, uint64_t seed, int mode,
+                                  int32_t* accepted_len, void* y_out, float* log_ratio_out,
+                                  float* delta_norm_out, uint32_t* status_out,
+                                  sdv_stream_t stream) {
+  const size_t need = sdv_workspace_bytes(B, L, d, dtype);
+  if (need == 0) return SDV_EINVAL;
+  if (need > (size_t)SDV_NOALLOC_SCRATCH_BYTES) return SDV_ENOWORKSPACE;
+  void* scratch = nullptr;
+  const int err = noalloc_scratch(&scratch);
+  if (err != 0) {
+    cudaGetLastError();  // reset the runtime's last-error slot so a later launch check does not report it
+    return SDV_ECUDA;
+  }
+  // The tickets that must start at zero are cleared by the call itself (a memset on
+  // `stream`); everything else in the workspace is written before it is read.
+  return sdv_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed, mode,
+                    accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, scratch,
+                    (size_t)SDV_NOALLOC_SCRATCH_BYTES, stream);
+}

@@ -13,6 +13,7 @@
 // Everything is fp32: GB300's fp64 rate is a small fraction of its fp32 rate.
 // The special-function helpers are __noinline__: inlined at every call site they
 // made the acceptance-scan kernel's code too large for the instruction cache.
+// Inside gdiff, g' stays inline so that its eight quadrature nodes interleave.
 // The forms below avoid the cancellations that fp32 would otherwise suffer:
 //  - v = alpha Phi(a+) - Phi(a-) is written as alpha Phi(a+) (1 - e^{x0}) with
 //    x0 = log(Phi(a-)/(alpha Phi(a+))) = g(a-) - g(a+), exact because
@@ -124,7 +125,7 @@ static __device__ __noinline__ float gfun(float a) {
 // error is damped by the levels above; only the final division is exact.  Deeper
 // levels are needed only near the switch point (16 levels give ~5e-10 at x = 4,
 // 8 levels ~4e-10 at x = 8).
-static __device__ __noinline__ float gprime(float s) {
+__device__ __forceinline__ float gprime(float s) {
   if (s < -4.0f) {
     const float x = -s;
     float acc = x;
@@ -261,8 +262,10 @@ struct USampleScratch {
 //  1. bracket: NT candidates t_k = s0 2^(k/8 - 8) (the paper's doubling of the
 //     bracket, eight steps per octave, all at once), s0 = 1/max(1, |a-|) the
 //     scale of the residual's spread;
-//  2. two rounds of NT-way multisection;
-//  3. a secant step between the bracket ends (g known there).
+//  2. one round of NT-way multisection;
+//  3. one Newton step from the bracket end with the smaller |g|, clamped to the
+//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form,
+//     log psi(a+ - t) = a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)).
 template <int NT>
 __device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits,
                                                uint32_t* status, USampleScratch* sm) {
@@ -301,8 +304,7 @@ __device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits
   float lo = (f == 0) ? 0.0f : sm->t[0];
   float glo = (f == 0) ? -INFINITY : sm->g[0];
   __syncthreads();
-#pragma unroll 1
-  for (int round = 0; round < 2; ++round) {
+  {
     const float h = (hi - lo) * (1.0f / (float)NT);
     const float t = (tid < NT - 1) ? lo + (float)(tid + 1) * h : hi;
     const float gt = (tid < NT - 1) ? gap(t) : ghi;
@@ -315,14 +317,18 @@ __device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits
     ghi = sm->g[1];
     __syncthreads();
   }
-  float t;
-  if (isfinite(glo) && isfinite(ghi) && ghi > glo) {
-    const float frac = fminf(fmaxf(-glo / (ghi - glo), 0.0f), 1.0f);
-    t = lo + frac * (hi - lo);
-  } else {
-    t = 0.5f * (lo + hi);
-  }
-  return P.ap - t;
+  // Newton step from the closer end
+  const bool from_lo = isfinite(glo) && (-glo < ghi);
+  const float te = from_lo ? lo : hi, ge = from_lo ? glo : ghi;
+  const float lpsi = P.am * te - 0.5f * te * te + logexpm1(P.D * te) - P.lvn;
+  const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
+  const float dg = expf(lpsi - lden);
+  // Return u directly: u_e = fl(a+ - t_e) is the point the evaluator used, so adding
+  // the Newton correction keeps U's rounding relative to |U| rather than to |a+|.
+  const float ue = P.ap - te;
+  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
+  step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
+  return ue + step;
 }
 
 // ---------------------------------------------------------------- element access

@@ -69,8 +69,9 @@ def test_usample_matches_oracle(api):
     Uo = OV.usample_bisection(D.astype(np.float64), la.astype(np.float64), OP.uniform_of(wb))
     err = np.abs(U - Uo)
     tol = 5e-6 + 3e-7 * np.abs(Uo)
-    assert np.all(err <= tol), "worst U error %g at D=%g la=%g" % (
-        err.max(), D[np.argmax(err - tol)], la[np.argmax(err - tol)])
+    i = int(np.argmax(err - tol))
+    assert np.all(err <= tol), "worst U error %g at D=%r la=%r w_bits=%d: gpu %r oracle %r" % (
+        err[i], float(D[i]), float(la[i]), int(wb[i]), float(U[i]), float(Uo[i]))
 
 
 def test_usample_degenerate_inputs(api):

@@ -1,0 +1,128 @@
+"""Pins for the fp64 sampler oracle: the VP schedule, the GMM score, the Euler-Maruyama
+chain and the speculative samplers (Free / Frozen drafter, sample / block verification).
+
+Independent references: quadrature of beta, finite differences of the mixture
+log-density (scipy), the closed-form law of the linear (one-component) chain, and the
+paper's remark that the Frozen drafter's first draft is always accepted.
+"""
+import math
+
+import numpy as np
+import pytest
+from scipy import integrate, stats
+from scipy.special import logsumexp
+
+from oracle import sampler as S
+from oracle import verify as V
+
+
+def _gmm(C, d, seed, comp_var=1.0, scale=2.0):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    means = scale * rng.standard_normal((C, d))
+    w = rng.dirichlet(np.ones(C))
+    return dict(means=means, log_weights=np.log(w), comp_var=comp_var)
+
+
+def test_alpha_bar_is_exp_of_integrated_beta():
+    sch = S.VPSchedule(K=100, churn=0.5)
+    for t in (1e-4, 0.1, 0.5, 0.93, 1.0):
+        ref = math.exp(-integrate.quad(lambda s: float(sch.beta(s)), 0, t)[0])
+        assert abs(float(sch.alpha_bar(t)) - ref) < 1e-12
+    # sigma_k = sqrt(delta) * churn * g_{1 - t_k}, g = sqrt(beta)
+    assert abs(float(sch.sigma(10)) - math.sqrt(0.01) * 0.5 * math.sqrt(float(sch.beta(0.9)))) < 1e-15
+    assert float(sch.tfwd(100)) == 1e-4
+
+
+def test_gmm_score_is_gradient_of_log_density():
+    sch = S.VPSchedule(K=100, churn=0.5)
+    gmm = _gmm(5, 4, 1)
+    rng = np.random.Generator(np.random.PCG64(2))
+
+    def logq(x, tf):
+        ab = float(sch.alpha_bar(tf))
+        v = ab * gmm["comp_var"] + 1 - ab
+        comps = [lw + stats.multivariate_normal.logpdf(x, math.sqrt(ab) * mu, v * np.eye(4))
+                 for lw, mu in zip(gmm["log_weights"], gmm["means"])]
+        return logsumexp(comps)
+
+    for tf in (0.02, 0.3, 0.9):
+        for _ in range(4):
+            x = 2.5 * rng.standard_normal(4)
+            s = S.gmm_score(x[None], np.array([tf]), gmm["means"], gmm["log_weights"],
+                            gmm["comp_var"], sch)[0]
+            h = 1e-5
+            fd = np.array([(logq(x + h * e, tf) - logq(x - h * e, tf)) / (2 * h) for e in np.eye(4)])
+            np.testing.assert_allclose(s, fd, rtol=1e-5, atol=1e-6)
+
+
+def _check_law(y, m, var, n_sigma=4.0):
+    n, d = y.shape
+    se_m = math.sqrt(var / n)
+    assert np.all(np.abs(y.mean(0) - m) < n_sigma * se_m), (y.mean(0), m)
+    se_v = var * math.sqrt(2.0 / (n - 1))
+    assert np.all(np.abs(y.var(0) - var) < n_sigma * se_v), (y.var(0), var)
+    for c in range(d):
+        assert stats.kstest((y[:, c] - m[c]) / math.sqrt(var), "norm").pvalue > 1e-3
+
+
+@pytest.fixture(scope="module", params=[40, 3])
+def linear_setup(request):
+    """K = 40 (many rounds) and K = 3 < L (a single window that reaches the end of
+    sampling, where a full accept must stop at yhat_K and take no bonus step)."""
+    sch = S.VPSchedule(K=request.param, churn=0.8)
+    gmm = dict(means=np.array([[1.5, -2.0, 0.5]]), log_weights=np.zeros(1), comp_var=0.5)
+    m, var = S.linear_gaussian_moments(gmm["means"][0], gmm["comp_var"], sch)
+    return sch, gmm, m, var
+
+
+def test_em_chain_matches_linear_closed_form(linear_setup):
+    sch, gmm, m, var = linear_setup
+    y = S.em_sample(20000, 3, gmm, sch, seed=3)
+    _check_law(y, m, var)
+
+
+@pytest.mark.parametrize("mode,drafter", [(V.MODE_SAMPLE, "free"), (V.MODE_BLOCK, "free"),
+                                          (V.MODE_BLOCK, "frozen")])
+def test_speculative_sampler_matches_linear_closed_form(linear_setup, mode, drafter):
+    """Exactness of the whole round (drafter, verification, residual, bonus, end handling,
+    score cache): Y_K has the law of the plain EM chain."""
+    sch, gmm, m, var = linear_setup
+    out = S.speculative_sample(20000, 3, 4, mode, gmm, sch, seed=4, drafter=drafter)
+    assert np.all(out["k"] == sch.K)
+    _check_law(out["y"], m, var)
+    assert 1 <= out["rounds"] <= sch.K
+
+
+def test_frozen_drafter_always_accepts_its_first_draft():
+    sch = S.VPSchedule(K=30, churn=0.5)
+    gmm = _gmm(3, 4, 5)
+    out = S.speculative_sample(300, 4, 4, V.MODE_SAMPLE, gmm, sch, seed=6, drafter="frozen")
+    for t in out["taus"]:
+        assert np.all((t == 0) | (t >= 2))
+
+
+def test_block_is_more_efficient_than_sample_on_the_mixture():
+    sch = S.VPSchedule(K=60, churn=0.5)
+    gmm = _gmm(4, 6, 7)
+    r = {m: S.speculative_sample(400, 6, 6, m, gmm, sch, seed=8) for m in (0, 1)}
+    # fewer rounds (parallel target calls) per chain with block verification
+    assert r[1]["chain_rounds"].mean() < r[0]["chain_rounds"].mean()
+    for m in (0, 1):
+        assert np.all(r[m]["k"] == sch.K)
+        taus = np.concatenate([t[t > 0] for t in r[m]["taus"]])
+        # every chain covers K steps: the taus of a chain sum to at least K
+        assert taus.sum() >= 400 * sch.K
+
+
+def test_speculative_and_em_agree_on_the_mixture():
+    """Two-sample checks between the speculative samplers and the plain chain (8 components)."""
+    sch = S.VPSchedule(K=50, churn=0.5)
+    gmm = _gmm(8, 4, 9)
+    n = 4000
+    y_em = S.em_sample(n, 4, gmm, sch, seed=10)
+    rng = np.random.Generator(np.random.PCG64(11))
+    dirs = rng.standard_normal((3, 4))
+    for mode in (V.MODE_SAMPLE, V.MODE_BLOCK):
+        y_sp = S.speculative_sample(n, 4, 5, mode, gmm, sch, seed=12)["y"]
+        for u in dirs:
+            assert stats.ks_2samp(y_em @ u, y_sp @ u).pvalue > 1e-3

@@ -231,6 +231,82 @@ int sdv_philox(const uint32_t *ctr, uint64_t seed, int n, uint32_t *out, sdv_str
 int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub,
                 float *out, sdv_stream_t stream);
 
+/* ---- end-to-end sampler on an analytic Gaussian-mixture target --------------
+ *
+ * Model (Eq. forward-process, backward-process, target-distribution): a
+ * variance-preserving forward SDE with beta(t) = beta_min + (beta_max - beta_min) t,
+ * f_t = -beta/2, g_t = sqrt(beta), abar_t = exp(-int_0^t beta); data distribution
+ * sum_c w_c N(mu_c, comp_var I) (means [C, d], log_weights [C], C <= SDV_MAX_COMPONENTS),
+ * so q_t = sum_c w_c N(sqrt(abar_t) mu_c, (abar_t comp_var + 1 - abar_t) I) with an exact
+ * score.  K generative steps, t_k = k/K, delta = 1/K, churn eps > 0:
+ *   m^q_k(y) = y + delta [beta/2 y + (1 + eps^2)/2 beta s_{1-t_k}(y)],
+ *   sigma_k = sqrt(delta) eps sqrt(beta), beta and s at forward time max(1 - t_k, t_floor).
+ * The Free drafter (Sec. "Self-Speculative Drafter") uses the same drift with the score
+ * kept from the previous round's parallel verification; the Frozen drafter
+ * (Eq. frozen-draft-drift) recomputes it at each round's start state.
+ * Random numbers: Y_0 from Philox stream 5 (seed), draft noise stream 4 with sub-counter =
+ * draft step (round seed), plain-chain noise stream 6 with sub-counter = k (seed); round r
+ * is keyed by the (r+1)-th SplitMix64 output of a stream started at `seed`.
+ */
+#define SDV_MAX_COMPONENTS 16
+#define SDV_DRAFTER_FREE   0
+#define SDV_DRAFTER_FROZEN 1
+
+/*
+ * sdv_gmm_target - the target call (the "target model" of Eq. target-distribution):
+ * for n state rows `states` [n, d] fp32 at generative steps k [n] (int32, 0 <= k <= K),
+ * writes m^q_k(state) to mq_out [n, d] and the score to score_out [n, d] (either may be
+ * NULL, not both).
+ */
+int sdv_gmm_target(const float *states, const int32_t *k, int n, int64_t d,
+                   const float *means, const float *log_weights, int C, float comp_var,
+                   int K, float churn, float beta_min, float beta_max, float t_floor,
+                   float *mq_out, float *score_out, sdv_stream_t stream);
+
+/*
+ * sdv_free_draft - the drafter: for chain b, gamma_b = L_eff[b] elementwise steps from
+ * y [B, d] starting at step k[b] with the cached score `score` [B, d]:
+ *   mu_draft[b, i] = m^p_{k+i}, x_draft[b, i] = yhat_{k+i+1} = m^p + sigma_{k+i} G_i,
+ *   sigma[b, i] = sigma_{k+i}, for i < gamma_b (other rows untouched).  G_i: stream 4,
+ * sub-counter i, key `seed`.  x_draft and mu_draft are [B, L, d]; sigma is [B, L].
+ */
+int sdv_free_draft(const float *y, const float *score, const int32_t *k, const int32_t *L_eff,
+                   int B, int L, int64_t d, int K, float churn, float beta_min, float beta_max,
+                   float t_floor, uint64_t seed, float *x_draft, float *mu_draft, float *sigma,
+                   sdv_stream_t stream);
+
+/* Bytes of device workspace sdv_sampler_run needs for (B, L, d); 0 for invalid sizes. */
+size_t sdv_sampler_workspace_bytes(int B, int L, int64_t d);
+
+/*
+ * sdv_sampler_run - speculative sampling of B chains (Alg. full-block-verification with
+ * the chosen drafter and verification mode) until every chain has reached step K or
+ * `max_rounds` rounds have run.  One round: gamma_k = min(L, K - k) draft steps, the
+ * parallel target call at yhat_k .. yhat_{k+gamma_k}, sdv_verify_ex (residual or bonus
+ * step), then k <- min(k + tau, K); a window that reaches K takes no bonus step.
+ * Unlike the other entry points this call synchronises: it enqueues the rounds on
+ * `stream` and reads the number of active chains back every 8 rounds.
+ *   y_out [B, d] fp32 out: the chains' states (Y_K when finished)
+ *   k_out [B], chain_rounds_out [B], tau_sum_out [B] int32 out or NULL: step reached,
+ *     rounds taken part in, sum of tau over those rounds
+ *   rounds_out: host int32 out, rounds run
+ */
+int sdv_sampler_run(int B, int L, int64_t d, const float *means, const float *log_weights, int C,
+                    float comp_var, int K, float churn, float beta_min, float beta_max,
+                    float t_floor, uint64_t seed, int mode, int drafter, int max_rounds,
+                    float *y_out, int32_t *k_out, int32_t *chain_rounds_out,
+                    int32_t *tau_sum_out, int32_t *rounds_out, void *workspace,
+                    size_t workspace_bytes, sdv_stream_t stream);
+
+/*
+ * sdv_em_sample - the plain (non-speculative) Euler-Maruyama chain, Y_{k+1} =
+ * m^q_k(Y_k) + sigma_k G_k for k = 0 .. K-1 from Y_0 (stream 5), G_k from stream 6 with
+ * sub-counter k; y_out [B, d] fp32 out.  K kernel launches on `stream`.
+ */
+int sdv_em_sample(int B, int64_t d, const float *means, const float *log_weights, int C,
+                  float comp_var, int K, float churn, float beta_min, float beta_max,
+                  float t_floor, uint64_t seed, float *y_out, sdv_stream_t stream);
+
 /*
  * Profiling aid (not part of the method): when enabled, every later
  * sdv_verify / sdv_verify_ex call made on this host thread records four CUDA

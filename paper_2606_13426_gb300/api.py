@@ -183,3 +183,74 @@ def normals(seed, Bn, d, stream_id, sub=0, device="cuda"):
     out = torch.empty(Bn, d, dtype=torch.float32, device=device)
     B.sdv_normals(int(seed) & 0xFFFFFFFFFFFFFFFF, Bn, d, stream_id, sub, _ptr(out), _stream())
     return out
+
+
+
+class GmmTarget:
+    """Analytic Gaussian-mixture target and its variance-preserving schedule (device copies)."""
+
+    def __init__(self, means, log_weights, comp_var, K, churn, beta_min=0.1, beta_max=20.0,
+                 t_floor=1e-4, device="cuda"):
+        self.means = torch.as_tensor(means, dtype=torch.float32).to(device).contiguous()
+        self.log_weights = torch.as_tensor(log_weights, dtype=torch.float32).to(device).contiguous()
+        self.C, self.d = self.means.shape
+        self.comp_var = float(comp_var)
+        self.K = int(K)
+        self.churn = float(churn)
+        self.beta_min, self.beta_max, self.t_floor = float(beta_min), float(beta_max), float(t_floor)
+
+    def sched(self):
+        return (self.K, self.churn, self.beta_min, self.beta_max, self.t_floor)
+
+    def params(self):
+        return (_ptr(self.means), _ptr(self.log_weights), self.C, self.comp_var) + self.sched()
+
+
+def gmm_target(states, k, target):
+    """m^q_k(state) and the score for rows of states [n, d] (sdv_gmm_target)."""
+    _need_cuda(states, k)
+    n, d = states.shape
+    mq = torch.empty_like(states)
+    sc = torch.empty_like(states)
+    B.sdv_gmm_target(_ptr(states), _ptr(k), n, d, *target.params(), _ptr(mq), _ptr(sc), _stream())
+    return mq, sc
+
+
+def free_draft(y, score, k, L_eff, L, target, seed):
+    """The drafter's gamma_b steps (sdv_free_draft): x_draft, mu_draft [B, L, d], sigma [B, L]."""
+    _need_cuda(y, score, k, L_eff)
+    Bn, d = y.shape
+    x = torch.zeros(Bn, L, d, dtype=torch.float32, device=y.device)
+    mp = torch.zeros_like(x)
+    sg = torch.zeros(Bn, L, dtype=torch.float32, device=y.device)
+    B.sdv_free_draft(_ptr(y), _ptr(score), _ptr(k), _ptr(L_eff), Bn, L, d, *target.sched(),
+                     int(seed) & 0xFFFFFFFFFFFFFFFF, _ptr(x), _ptr(mp), _ptr(sg), _stream())
+    return x, mp, sg
+
+
+def sampler_run(Bn, L, target, seed, mode="block", drafter="free", max_rounds=None,
+                workspace=None):
+    """Speculative sampling of Bn chains to step K (sdv_sampler_run); returns a dict."""
+    dev = target.means.device
+    d = target.d
+    if workspace is None:
+        workspace = torch.empty(B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8,
+                                device=dev)
+    y = torch.empty(Bn, d, dtype=torch.float32, device=dev)
+    k = torch.empty(Bn, dtype=torch.int32, device=dev)
+    cr = torch.empty(Bn, dtype=torch.int32, device=dev)
+    ts = torch.empty(Bn, dtype=torch.int32, device=dev)
+    dr = {"free": B.SDV_DRAFTER_FREE, "frozen": B.SDV_DRAFTER_FROZEN}[drafter]
+    mr = target.K if max_rounds is None else int(max_rounds)
+    rounds = B.sdv_sampler_run(Bn, L, d, *target.params(), int(seed) & 0xFFFFFFFFFFFFFFFF,
+                               _MODES[mode], dr, mr, _ptr(y), _ptr(k), _ptr(cr), _ptr(ts),
+                               _ptr(workspace), workspace.numel(), _stream())
+    return dict(y=y, k=k, chain_rounds=cr, tau_sum=ts, rounds=rounds)
+
+
+def em_sample(Bn, target, seed):
+    """The plain Euler-Maruyama chain (sdv_em_sample)."""
+    y = torch.empty(Bn, target.d, dtype=torch.float32, device=target.means.device)
+    B.sdv_em_sample(Bn, target.d, *target.params(), int(seed) & 0xFFFFFFFFFFFFFFFF, _ptr(y),
+                    _stream())
+    return y

@@ -27,6 +27,9 @@ SDV_STATUS_ZERO_DELTA = 1
 SDV_STATUS_NONFINITE = 2
 SDV_STATUS_USAMPLE_RANGE = 4
 SDV_MAX_L = 64
+SDV_MAX_COMPONENTS = 16
+SDV_DRAFTER_FREE = 0
+SDV_DRAFTER_FROZEN = 1
 SDV_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 _P = ctypes.c_void_p
@@ -55,6 +58,13 @@ SIGNATURES = {
     "sdv_usample": (_I, [_P, _P, _P, _I, _P, _P, _P]),
     "sdv_philox": (_I, [_P, _U64, _I, _P, _P]),
     "sdv_normals": (_I, [_U64, _I, _I64, _I, _U32, _P, _P]),
+    "sdv_gmm_target": (_I, [_P, _P, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _P, _P, _P]),
+    "sdv_free_draft": (_I, [_P, _P, _P, _P, _I, _I, _I64, _I, _F, _F, _F, _F, _U64, _P, _P, _P,
+                            _P]),
+    "sdv_sampler_workspace_bytes": (_SZ, [_I, _I, _I64]),
+    "sdv_sampler_run": (_I, [_I, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _I, _I, _I,
+                             _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "sdv_em_sample": (_I, [_I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _P, _P]),
     "sdv_timing_enable": (_I, [_I]),
     "sdv_timing_read": (_I, [_I, _P]),
 }
@@ -177,3 +187,36 @@ def sdv_timing_read(n_calls):
     ms = (ctypes.c_float * 3)()
     _call("sdv_timing_read", n_calls, ctypes.addressof(ms))
     return [float(v) for v in ms]
+
+
+def sdv_gmm_target(states, k, n, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max,
+                   t_floor, mq_out, score_out, stream):
+    return _call("sdv_gmm_target", states, k, n, d, means, log_weights, C, comp_var, K, churn,
+                 beta_min, beta_max, t_floor, mq_out, score_out, stream)
+
+
+def sdv_free_draft(y, score, k, L_eff, B, L, d, K, churn, beta_min, beta_max, t_floor, seed,
+                   x_draft, mu_draft, sigma, stream):
+    return _call("sdv_free_draft", y, score, k, L_eff, B, L, d, K, churn, beta_min, beta_max,
+                 t_floor, seed, x_draft, mu_draft, sigma, stream)
+
+
+def sdv_sampler_workspace_bytes(B, L, d):
+    return int(load().sdv_sampler_workspace_bytes(B, L, d))
+
+
+def sdv_sampler_run(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max,
+                    t_floor, seed, mode, drafter, max_rounds, y_out, k_out, chain_rounds_out,
+                    tau_sum_out, workspace, workspace_bytes, stream):
+    """Returns the number of rounds run (the C call's rounds_out)."""
+    rounds = ctypes.c_int32(0)
+    _call("sdv_sampler_run", B, L, d, means, log_weights, C, comp_var, K, churn, beta_min,
+          beta_max, t_floor, seed, mode, drafter, max_rounds, y_out, k_out, chain_rounds_out,
+          tau_sum_out, ctypes.addressof(rounds), workspace, workspace_bytes, stream)
+    return int(rounds.value)
+
+
+def sdv_em_sample(B, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max, t_floor,
+                  seed, y_out, stream):
+    return _call("sdv_em_sample", B, d, means, log_weights, C, comp_var, K, churn, beta_min,
+                 beta_max, t_floor, seed, y_out, stream)

@@ -79,4 +79,10 @@ struct WsLayout {
 
 WsLayout ws_layout(int B, int L, int64_t d, int dtype);
 
+// Records a cudaError_t for sdv_last_cuda_error() (this host thread).
+void set_last_cuda_error(int err);
+
+// Largest number of mixture components of the analytic target.
+constexpr int kSdvMaxComponents = SDV_MAX_COMPONENTS;
+
 }  // namespace sdv

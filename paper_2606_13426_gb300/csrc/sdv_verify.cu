@@ -670,6 +670,8 @@ __global__ void k_normals(uint64_t seed, int B, int64_t d, uint32_t stream, uint
 // ---------------------------------------------------------------- host side
 static thread_local int g_last_cuda_error = 0;
 
+void set_last_cuda_error(int err) { g_last_cuda_error = err; }
+
 static int check_launch() {
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {

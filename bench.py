@@ -45,7 +45,9 @@ def parse():
     p.add_argument("--steps", type=int, default=20000)
     p.add_argument("--warmup", type=int, default=50)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="pixel", choices=["pixel", "latent", "highres"])
+    p.add_argument("--workload", default="pixel", choices=["pixel", "latent", "highres", "sampler"])
+    p.add_argument("--sampler-L", default="4,8,16",
+                   help="draft windows of the end-to-end sampler workload")
     p.add_argument("--mode", default="block", choices=["block", "sample"])
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -207,11 +209,69 @@ def run_reference(args, world, rank):
     print(json.dumps(line))
 
 
+def run_sampler(args, world, rank, local):
+    """End-to-end speculative sampler on the analytic 8-component mixture (B = 1024 chains,
+    d = 1024, K = 1000 VP Euler-Maruyama steps, churn 0.5, Free drafter) against the plain
+    Euler-Maruyama chain: wall-clock, rounds and accepted steps per parallel target call."""
+    import torch
+    import __graft_entry__ as G
+    G.build()
+    from paper_2606_13426_gb300 import api
+    torch.cuda.set_device(local)
+    cfg = W.SAMPLER_CONFIG
+    gm = W.make_gmm()
+    tgt = api.GmmTarget(torch.from_numpy(gm["means"]), torch.from_numpy(gm["log_weights"]),
+                        gm["comp_var"], cfg["K"], cfg["churn"])
+    Bn, d, K = cfg["B"], cfg["d"], cfg["K"]
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        out = fn()
+        torch.cuda.synchronize()
+        return out, time.perf_counter() - t0
+
+    timed(lambda: api.em_sample(Bn, tgt, 1))
+    t_em = min(timed(lambda: api.em_sample(Bn, tgt, 1 + i))[1] for i in range(3))
+    runs = {}
+    for L in [int(v) for v in args.sampler_L.split(",")]:
+        ws = torch.empty(api.B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8, device="cuda")
+        for mode in ("sample", "block"):
+            timed(lambda: api.sampler_run(Bn, L, tgt, 7, mode, workspace=ws))
+            best = None
+            for i in range(3):
+                r, t = timed(lambda: api.sampler_run(Bn, L, tgt, 100 + i, mode, workspace=ws))
+                if best is None or t < best[1]:
+                    best = (r, t)
+            r, t = best
+            cr = r["chain_rounds"].cpu().numpy().astype(np.float64)
+            ts = r["tau_sum"].cpu().numpy().astype(np.float64)
+            runs["L%d_%s" % (L, mode)] = {
+                "ms": 1e3 * t, "rounds": r["rounds"], "mean_chain_rounds": float(cr.mean()),
+                "mean_tau": float(ts.sum() / cr.sum()),
+                "target_calls_per_chain": float(cr.mean() + 1.0),
+                "speedup_vs_em": t_em / t}
+    best_key = min(runs, key=lambda k2: runs[k2]["ms"])
+    line = {
+        "metric": "end-to-end speculative sampler: denoising steps/s; mean accepted steps/target call",
+        "value": Bn * K / (runs[best_key]["ms"] * 1e-3), "unit": "denoising steps/s",
+        "n_gpus": 1, "higher_is_better": True, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "analytic 8-component GMM, d=%d, B=%d, K=%d VP EM steps, churn %.2f, "
+                               "Free drafter" % (d, Bn, K, cfg["churn"]), "best": best_key},
+        "em_ms": 1e3 * t_em, "em_steps_per_s": Bn * K / t_em, "runs": runs,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+
+
 def main():
     args = parse()
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.workload == "sampler":
+        run_sampler(args, world, rank, local)
         return
 
     import torch

@@ -46,17 +46,24 @@ struct Gmm {
   float comp_var;
 };
 
-constexpr int kGmmThreads = 256;
+constexpr int kGmmThreads = 256;              // 8 warps, one state row per warp at a time
+constexpr int kGmmWarps = kGmmThreads / 32;
+constexpr size_t kGmmSmemCap = 96 * 1024;     // stage the means in shared memory up to this size
 
-// m^q and the score for one state row z (generative step k), by the whole CTA.
-// mq / score may be null.  z may alias mq (each element is read before it is written
-// by the same thread), which the in-place EM step uses.
-__device__ void gmm_row(const float* z, int64_t d, int k, const Sched& S, const Gmm& G,
-                        float* mq, float* score, float add_sigma, uint64_t noise_seed,
-                        uint32_t noise_chain, uint32_t noise_stream, uint32_t noise_sub) {
-  __shared__ float red[kGmmThreads / 32][kSdvMaxComponents];
-  __shared__ float d2s[kSdvMaxComponents];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+// m^q and the score for one state row z (generative step k), by one warp.  mu points to
+// the means [C, d] (shared or global memory).  mq / score may be null; z may alias mq:
+// each lane reads a group of four elements before it writes it, and no other lane
+// touches that group.  add_sigma != 0 adds sigma * G (Philox stream noise_stream,
+// sub-counter noise_sub; one Philox block per group of four) to mq.
+// VEC: d % 4 == 0 and 16-byte aligned rows (float4 accesses); MAXC >= C components.
+template <int MAXC, bool VEC>
+__device__ __forceinline__ void gmm_row_warp(const float* z, int64_t d, int k, const Sched& S,
+                                             const Gmm& G, const float* mu, float* mq, float* score,
+                                             float add_sigma, uint64_t noise_seed,
+                                             uint32_t noise_chain, uint32_t noise_stream,
+                                             uint32_t noise_sub) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
   const int C = G.C;
   const float tf = S.tfwd(k);
   const float ab = S.abar(tf);
@@ -64,101 +71,146 @@ __device__ void gmm_row(const float* z, int64_t d, int k, const Sched& S, const 
   const float v = ab * G.comp_var + 1.0f - ab;
   const float b = S.beta(tf);
   const float cst = 0.5f * (1.0f + S.churn * S.churn);
-  // pass 1: squared distances to the scaled centres
-  float acc[kSdvMaxComponents];
+  const int64_t ng = (d + 3) / 4;
+  auto load_group = [&](const float* p, int64_t gi, float (&f)[4]) {
+    if (VEC) {
+      const float4 t = *reinterpret_cast<const float4*>(p + 4 * gi);
+      f[0] = t.x; f[1] = t.y; f[2] = t.z; f[3] = t.w;
+    } else {
 #pragma unroll
-  for (int c = 0; c < kSdvMaxComponents; ++c) acc[c] = 0.f;
-  for (int64_t i = tid; i < d; i += kGmmThreads) {
-    const float zi = z[i];
+      for (int q = 0; q < 4; ++q) f[q] = (4 * gi + q < d) ? p[4 * gi + q] : 0.f;
+    }
+  };
+  // pass 1: squared distances to the scaled centres sqrt(abar) mu_c
+  float acc[MAXC];
 #pragma unroll
-    for (int c = 0; c < kSdvMaxComponents; ++c) {
+  for (int c = 0; c < MAXC; ++c) acc[c] = 0.f;
+#pragma unroll 4
+  for (int64_t gi = lane; gi < ng; gi += 32) {
+    float zf[4];
+    load_group(z, gi, zf);
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) {
       if (c < C) {
-        const float df = zi - sab * __ldg(G.means + (int64_t)c * d + i);
-        acc[c] = fmaf(df, df, acc[c]);
+        float mf[4];
+        load_group(mu + (int64_t)c * d, gi, mf);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float df = (4 * gi + q < d) ? zf[q] - sab * mf[q] : 0.f;
+          acc[c] = fmaf(df, df, acc[c]);
+        }
       }
     }
   }
-#pragma unroll
-  for (int c = 0; c < kSdvMaxComponents; ++c) {
-    if (c < C) {
-      float a = acc[c];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(0xffffffffu, a, o);
-      if (lane == 0) red[warp][c] = a;
-    }
-  }
-  __syncthreads();
-  if (tid < C) {
-    float a = 0.f;
-    for (int w = 0; w < kGmmThreads / 32; ++w) a += red[w][tid];
-    d2s[tid] = a;
-  }
-  __syncthreads();
-  // responsibilities r_c = softmax(log w_c - d2_c / (2 v))
-  float r[kSdvMaxComponents];
+  // responsibilities r_c = softmax(log w_c - d2_c / (2 v)), identical in every lane
+  float r[MAXC];
   float mx = -INFINITY;
 #pragma unroll
-  for (int c = 0; c < kSdvMaxComponents; ++c) {
-    r[c] = (c < C) ? __ldg(G.log_w + c) - d2s[c] / (2.0f * v) : -INFINITY;
+  for (int c = 0; c < MAXC; ++c) {
+    float a = acc[c];
+    if (c < C) {
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(FULL, a, o);
+    }
+    r[c] = (c < C) ? __ldg(G.log_w + c) - a / (2.0f * v) : -INFINITY;
     mx = fmaxf(mx, r[c]);
   }
   float den = 0.f;
 #pragma unroll
-  for (int c = 0; c < kSdvMaxComponents; ++c) {
+  for (int c = 0; c < MAXC; ++c) {
     r[c] = (c < C) ? expf(r[c] - mx) : 0.f;
     den += r[c];
   }
-  const float inv = 1.0f / den;
-  // pass 2: score and target mean (optionally plus sigma * noise)
-  for (int64_t i0 = 4 * (int64_t)tid; i0 < d; i0 += 4 * kGmmThreads) {
+  const float w_sc = sab / den;  // folds the softmax normaliser and sqrt(abar)
+  // pass 2: score and target mean
+#pragma unroll 4
+  for (int64_t gi = lane; gi < ng; gi += 32) {
+    float zf[4], wsum[4] = {0.f, 0.f, 0.f, 0.f};
+    load_group(z, gi, zf);
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) {
+      if (c < C) {
+        float mf[4];
+        load_group(mu + (int64_t)c * d, gi, mf);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) wsum[q] = fmaf(r[c], mf[q], wsum[q]);
+      }
+    }
     float G4[4] = {0.f, 0.f, 0.f, 0.f};
     if (add_sigma != 0.f) {
-      const float4 n4 = normals4(noise_seed, noise_chain, (uint32_t)(i0 / 4), noise_stream, noise_sub);
+      const float4 n4 = normals4(noise_seed, noise_chain, (uint32_t)gi, noise_stream, noise_sub);
       G4[0] = n4.x; G4[1] = n4.y; G4[2] = n4.z; G4[3] = n4.w;
     }
+    float sc[4], m[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const int64_t i = i0 + q;
-      if (i >= d) break;
-      const float zi = z[i];
-      float wsum = 0.f;
+      sc[q] = (w_sc * wsum[q] - zf[q]) / v;
+      m[q] = zf[q] + S.delta * (0.5f * b * zf[q] + cst * b * sc[q]) + add_sigma * G4[q];
+    }
+    if (VEC) {
+      if (score) *reinterpret_cast<float4*>(score + 4 * gi) = make_float4(sc[0], sc[1], sc[2], sc[3]);
+      if (mq) *reinterpret_cast<float4*>(mq + 4 * gi) = make_float4(m[0], m[1], m[2], m[3]);
+    } else {
 #pragma unroll
-      for (int c = 0; c < kSdvMaxComponents; ++c)
-        if (c < C) wsum = fmaf(r[c], __ldg(G.means + (int64_t)c * d + i), wsum);
-      const float sc = (sab * wsum * inv - zi) / v;
-      const float m = zi + S.delta * (0.5f * b * zi + cst * b * sc);
-      if (score) score[i] = sc;
-      if (mq) mq[i] = m + add_sigma * G4[q];
+      for (int q = 0; q < 4; ++q) {
+        if (4 * gi + q < d) {
+          if (score) score[4 * gi + q] = sc[q];
+          if (mq) mq[4 * gi + q] = m[q];
+        }
+      }
     }
   }
 }
 
-// Target means and scores for rows of a [n, d] array at steps k[row]; rows whose
-// window mask (if given) is 0 are skipped.
-__global__ void __launch_bounds__(kGmmThreads)
-k_gmm_rows(const float* __restrict__ states, const int32_t* __restrict__ k, const int32_t* __restrict__ mask,
-           int64_t d, Sched S, Gmm G, float* mq, float* score) {
-  const int row = blockIdx.x;
-  if (mask && mask[row] == 0) return;
-  const int64_t o = (int64_t)row * d;
-  gmm_row(states + o, d, k[row], S, G, mq ? mq + o : nullptr, score ? score + o : nullptr, 0.f, 0,
-          0, 0, 0);
+// Stage the means in dynamic shared memory (when the launch gave it room); returns the
+// pointer the warps read from.
+__device__ __forceinline__ const float* stage_means(const Gmm& G, int64_t d, bool use_smem) {
+  extern __shared__ float mu_s[];
+  if (!use_smem) return G.means;
+  const int64_t n = (int64_t)G.C * d;
+  for (int64_t i = threadIdx.x; i < n; i += blockDim.x) mu_s[i] = __ldg(G.means + i);
+  __syncthreads();
+  return mu_s;
 }
 
-// Parallel target call of a round: state j of chain b is y[b] (j = 0) or x_draft[b, j-1],
-// at step k[b] + j, for j = 0 .. gamma_b.  Means go to mu_target[b, j] (j < gamma_b) or
-// mu_bonus[b] (j = gamma_b, with sigma_bonus[b] = sigma_{k+gamma}); scores to sc_all[b, j].
+// Target means and scores for rows of a [n, d] array at steps k[row]; one warp per row;
+// rows whose window mask (if given) is 0 are skipped.
+template <int MAXC, bool VEC>
+__global__ void __launch_bounds__(kGmmThreads)
+k_gmm_rows(const float* __restrict__ states, const int32_t* __restrict__ k, const int32_t* __restrict__ mask,
+           int n, int64_t d, Sched S, Gmm G, bool use_smem, float* mq, float* score) {
+  const float* mu = stage_means(G, d, use_smem);
+  const int warp = threadIdx.x >> 5;
+  for (int row = blockIdx.x * kGmmWarps + warp; row < n; row += gridDim.x * kGmmWarps) {
+    if (mask && mask[row] == 0) continue;
+    const int64_t o = (int64_t)row * d;
+    gmm_row_warp<MAXC, VEC>(states + o, d, k[row], S, G, mu, mq ? mq + o : nullptr,
+                            score ? score + o : nullptr, 0.f, 0, 0, 0, 0);
+  }
+}
+
+// Parallel target call of a round, one CTA per chain: state j of chain b is y[b] (j = 0)
+// or x_draft[b, j-1], at step k[b] + j, for j = 0 .. gamma_b.  Means go to mu_target[b, j]
+// (j < gamma_b) or mu_bonus[b] (j = gamma_b, with sigma_bonus[b] = sigma_{k+gamma});
+// scores to sc_all[b, j].
+template <int MAXC, bool VEC>
 __global__ void __launch_bounds__(kGmmThreads)
 k_round_target(const float* __restrict__ y, const float* __restrict__ x_draft,
                const int32_t* __restrict__ kk, const int32_t* __restrict__ gam, int L, int64_t d,
-               Sched S, Gmm G, float* mu_target, float* mu_bonus, float* sigma_bonus, float* sc_all) {
-  const int b = blockIdx.x / (L + 1), j = blockIdx.x - b * (L + 1);
+               Sched S, Gmm G, bool use_smem, float* mu_target, float* mu_bonus, float* sigma_bonus,
+               float* sc_all) {
+  const int b = blockIdx.x;
   const int g = gam[b];
-  if (g == 0 || j > g) return;
-  const float* z = (j == 0) ? y + (int64_t)b * d : x_draft + ((int64_t)b * L + j - 1) * d;
-  float* mq = (j < g) ? mu_target + ((int64_t)b * L + j) * d : mu_bonus + (int64_t)b * d;
-  gmm_row(z, d, kk[b] + j, S, G, mq, sc_all + ((int64_t)b * (L + 1) + j) * d, 0.f, 0, 0, 0, 0);
-  if (j == g && threadIdx.x == 0) sigma_bonus[b] = S.sigma(kk[b] + g);
+  if (g == 0) return;  // CTA-uniform: before any barrier
+  const float* mu = stage_means(G, d, use_smem);
+  const int warp = threadIdx.x >> 5;
+  for (int j = warp; j <= g; j += kGmmWarps) {
+    const float* z = (j == 0) ? y + (int64_t)b * d : x_draft + ((int64_t)b * L + j - 1) * d;
+    float* mq = (j < g) ? mu_target + ((int64_t)b * L + j) * d : mu_bonus + (int64_t)b * d;
+    gmm_row_warp<MAXC, VEC>(z, d, kk[b] + j, S, G, mu, mq, sc_all + ((int64_t)b * (L + 1) + j) * d,
+                            0.f, 0, 0, 0, 0);
+  }
+  if (threadIdx.x == 0) sigma_bonus[b] = S.sigma(kk[b] + g);
 }
 
 // Free / Frozen drafter: gamma_b elementwise steps from y[b] with the cached score.
@@ -256,13 +308,63 @@ k_sampler_init(int B, int L, int64_t d, int K, uint64_t seed, float* y, int32_t*
   }
 }
 
-// One plain Euler-Maruyama step for every chain, in place: y <- m^q_k(y) + sigma_k G_k.
+// One plain Euler-Maruyama step for every chain, in place: y <- m^q_k(y) + sigma_k G_k;
+// one warp per chain.
+template <int MAXC, bool VEC>
 __global__ void __launch_bounds__(kGmmThreads)
-k_em_step(float* y, int64_t d, int k, Sched S, Gmm G, uint64_t seed) {
-  const int b = blockIdx.x;
-  float* row = y + (int64_t)b * d;
-  gmm_row(row, d, k, S, G, row, nullptr, S.sigma(k), seed, (uint32_t)b, kStreamEM, (uint32_t)k);
+k_em_step(float* y, int B, int64_t d, int k, Sched S, Gmm G, bool use_smem, uint64_t seed) {
+  const float* mu = stage_means(G, d, use_smem);
+  const int warp = threadIdx.x >> 5;
+  for (int b = blockIdx.x * kGmmWarps + warp; b < B; b += gridDim.x * kGmmWarps) {
+    float* row = y + (int64_t)b * d;
+    gmm_row_warp<MAXC, VEC>(row, d, k, S, G, mu, row, nullptr, S.sigma(k), seed, (uint32_t)b, kStreamEM,
+                            (uint32_t)k);
+  }
 }
+
+// Launch geometry of the one-warp-per-row kernels: dynamic shared memory for the means
+// when they fit, the component bound, vector accesses, and the grid for n rows.
+struct GmmLaunch {
+  bool smem;
+  size_t smem_bytes;
+  bool vec;
+  int maxc;
+};
+
+template <int MAXC, bool VEC>
+static void gmm_set_smem(size_t bytes) {
+  cudaFuncSetAttribute(k_gmm_rows<MAXC, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  cudaFuncSetAttribute(k_round_target<MAXC, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  cudaFuncSetAttribute(k_em_step<MAXC, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+// rows_aligned: every state / output row the kernel touches starts on a 16-byte boundary
+static GmmLaunch gmm_launch(int C, int64_t d, const void* means, bool rows_aligned) {
+  GmmLaunch g{};
+  const size_t bytes = (size_t)C * (size_t)d * sizeof(float);
+  g.smem = bytes <= kGmmSmemCap;
+  g.smem_bytes = g.smem ? bytes : 0;
+  g.vec = (d % 4 == 0) && (reinterpret_cast<uintptr_t>(means) % 16 == 0) && rows_aligned;
+  g.maxc = C <= 8 ? 8 : 16;
+  if (g.smem_bytes > 48 * 1024) {
+    if (g.maxc == 8) { gmm_set_smem<8, true>(g.smem_bytes); gmm_set_smem<8, false>(g.smem_bytes); }
+    else { gmm_set_smem<16, true>(g.smem_bytes); gmm_set_smem<16, false>(g.smem_bytes); }
+  }
+  return g;
+}
+
+static unsigned rows_grid(int n) { return (unsigned)std::max(1, (n + kGmmWarps - 1) / kGmmWarps); }
+
+#define SDV_GMM_DISPATCH(GL, KERNEL, GRID, STREAM, ...)                                          \
+  do {                                                                                          \
+    if ((GL).maxc == 8) {                                                                       \
+      if ((GL).vec) KERNEL<8, true><<<GRID, kGmmThreads, (GL).smem_bytes, STREAM>>>(__VA_ARGS__);  \
+      else KERNEL<8, false><<<GRID, kGmmThreads, (GL).smem_bytes, STREAM>>>(__VA_ARGS__);          \
+    } else {                                                                                    \
+      if ((GL).vec) KERNEL<16, true><<<GRID, kGmmThreads, (GL).smem_bytes, STREAM>>>(__VA_ARGS__); \
+      else KERNEL<16, false><<<GRID, kGmmThreads, (GL).smem_bytes, STREAM>>>(__VA_ARGS__);         \
+    }                                                                                           \
+  } while (0)
 
 static int launch_check() {
   const cudaError_t e = cudaGetLastError();
@@ -343,7 +445,12 @@ int sdv_gmm_target(const float* states, const int32_t* k, int n, int64_t d, cons
   if (n == 0) return SDV_OK;
   const Sched S = make_sched(K, churn, beta_min, beta_max, t_floor);
   const Gmm G{means, log_weights, C, comp_var};
-  k_gmm_rows<<<n, kGmmThreads, 0, (cudaStream_t)stream>>>(states, k, nullptr, d, S, G, mq_out, score_out);
+  // float4 paths need 16-byte aligned rows in every array the kernel touches
+  const bool al = ((reinterpret_cast<uintptr_t>(states) | reinterpret_cast<uintptr_t>(mq_out) |
+                    reinterpret_cast<uintptr_t>(score_out)) % 16) == 0;
+  const GmmLaunch gl = gmm_launch(C, d, means, al);
+  SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(n), (cudaStream_t)stream, states, k, nullptr, n, d, S, G,
+                   gl.smem, mq_out, score_out);
   return launch_check();
 }
 
@@ -405,12 +512,14 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
   const Gmm G{means, log_weights, C, comp_var};
   const int64_t ng = (int64_t)B * ((d + 3) / 4);
   const unsigned eg = (unsigned)((ng + 255) / 256);
+  // workspace arrays start on 256-byte boundaries
+  const GmmLaunch gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(workspace) % 16 == 0);
 
   int rc;
   k_sampler_init<<<eg, 256, 0, s>>>(B, L, d, K, seed, y, kk, gam, rounds, tsum);
   if ((rc = launch_check()) != SDV_OK) return rc;
   // the only explicit target call: the score at Y_0 (step 0)
-  k_gmm_rows<<<B, kGmmThreads, 0, s>>>(y, kk, nullptr, d, S, G, nullptr, sc);
+  SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), s, y, kk, nullptr, B, d, S, G, gl.smem, nullptr, sc);
   if ((rc = launch_check()) != SDV_OK) return rc;
 
   int r = 0;
@@ -418,12 +527,12 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
   for (; r < max_rounds; ++r) {
     const uint64_t seed_r = round_seed(seed, r);
     if (drafter == SDV_DRAFTER_FROZEN) {  // a fresh score at the round's start state
-      k_gmm_rows<<<B, kGmmThreads, 0, s>>>(y, kk, gam, d, S, G, nullptr, sc);
+      SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), s, y, kk, gam, B, d, S, G, gl.smem, nullptr, sc);
       if ((rc = launch_check()) != SDV_OK) return rc;
     }
     k_draft<<<eg, 256, 0, s>>>(y, sc, kk, gam, B, L, d, S, seed_r, xd, mpd, sg);
     if ((rc = launch_check()) != SDV_OK) return rc;
-    k_round_target<<<B * (L + 1), kGmmThreads, 0, s>>>(y, xd, kk, gam, L, d, S, G, mqd, mqb, sgb, scall);
+    SDV_GMM_DISPATCH(gl, k_round_target, B, s, y, xd, kk, gam, L, d, S, G, gl.smem, mqd, mqb, sgb, scall);
     if ((rc = launch_check()) != SDV_OK) return rc;
     rc = sdv_verify_ex(xd, mqd, mpd, sg, L, B, L, d, SDV_F32, seed_r, mode, gam, mqb, sgb,
                        SDV_RESIDUAL_DECOMPOSITION, 1.0f, acc, yo, nullptr, nullptr, nullptr, nullptr,
@@ -471,8 +580,9 @@ int sdv_em_sample(int B, int64_t d, const float* means, const float* log_weights
                                                               nullptr, nullptr);
   int rc = launch_check();
   if (rc != SDV_OK) return rc;
+  const GmmLaunch gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(y_out) % 16 == 0);
   for (int k = 0; k < K; ++k) {
-    k_em_step<<<B, kGmmThreads, 0, s>>>(y_out, d, k, S, G, seed);
+    SDV_GMM_DISPATCH(gl, k_em_step, rows_grid(B), s, y_out, B, d, k, S, G, gl.smem, seed);
     if ((rc = launch_check()) != SDV_OK) return rc;
   }
   return SDV_OK;

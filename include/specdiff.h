@@ -171,7 +171,7 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  *     own stream, but calls that overlap on the GPU (other streams, other host
  *     threads, same device) race on the array.  Serialise them, e.g. on one stream.
  */
-#define SDV_NOALLOC_SCRATCH_BYTES (1u << 20)
+#define SDV_NOALLOC_SCRATCH_BYTES (1u << 22)
 int sdv_verify_noalloc(const void *x_draft, const void *mu_target, const void *mu_draft,
                        const float *sigma, int64_t sigma_stride_b,
                        int B, int L, int64_t d, int dtype,

@@ -30,7 +30,7 @@ SDV_MAX_L = 64
 SDV_MAX_COMPONENTS = 16
 SDV_DRAFTER_FREE = 0
 SDV_DRAFTER_FROZEN = 1
-SDV_NOALLOC_SCRATCH_BYTES = 1 << 20
+SDV_NOALLOC_SCRATCH_BYTES = 1 << 22
 
 _P = ctypes.c_void_p
 _I = ctypes.c_int

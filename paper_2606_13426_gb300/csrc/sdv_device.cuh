@@ -6,9 +6,10 @@
 //    g'(s) = lambda(s) + s (lambda = phi/Phi, the inverse Mills ratio), and
 //    differences g(hi) - g(hi - h) by 8-point Gauss-Legendre quadrature.
 //  * The block-verification acceptance probability h_j (Algorithm
-//    block-verification) in log form (App. "Density ratio calculations").
+//    block-verification) in log form (App. "Density ratio calculations"), from
+//    the same residual mass log v that the U-sampler's setup computes.
 //  * The residual's 1-D draw U = Psi_alpha^{-1}(w) (Prop. decomposition,
-//    Eq. u-cdf, Algorithm u-sample) as a warp-cooperative multisection.
+//    Eq. u-cdf, Algorithm u-sample) as a one-warp multisection.
 //
 // Everything is fp32: GB300's fp64 rate is a small fraction of its fp32 rate.
 // The special-function helpers are __noinline__: inlined at every call site they
@@ -26,6 +27,19 @@
 //    Laplace's continued fraction for the Mills ratio with its first term
 //    cancelled analytically.
 #pragma once
+
+// Linkage of the special-function helpers (see above); a translation unit may
+// define SDV_HELPER before including this header.
+#ifndef SDV_HELPER
+#define SDV_HELPER __noinline__
+#endif
+// Unrolling of the quadrature nodes in gdiff (code size against node interleaving).
+#ifndef SDV_GL_UNROLL
+#define SDV_GL_UNROLL 8
+#endif
+namespace sdv {
+constexpr int kGLUnroll = SDV_GL_UNROLL;
+}
 
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -75,9 +89,11 @@ __device__ __forceinline__ uint4 philox_block(uint64_t seed, uint32_t c0, uint32
 
 // log u for u = (x + 1/2) 2^-32; the upper half goes through 1 - u, which is
 // exact in the integer domain, so log u keeps full relative accuracy near 1.
+// Both forms are evaluated and one selected (no divergence between lanes).
 __device__ __forceinline__ float log_uniform(uint32_t x) {
-  if (x < 0x80000000u) return logf(((float)x + 0.5f) * 0x1p-32f);
-  return log1pf(-(((float)(0xFFFFFFFFu - x) + 0.5f) * 0x1p-32f));
+  const float lo = logf(((float)x + 0.5f) * 0x1p-32f);
+  const float hi = log1pf(-(((float)(0xFFFFFFFFu - x) + 0.5f) * 0x1p-32f));
+  return (x < 0x80000000u) ? lo : hi;
 }
 
 // Box-Muller on two words: (r cos 2 pi u1, r sin 2 pi u1), r = sqrt(-2 ln u0).
@@ -108,37 +124,44 @@ static __constant__ float kGLx[4] = {0.18343464249564978f, 0.52553240991632899f,
 static __constant__ float kGLw[4] = {0.36268378337836166f, 0.31370664587788688f,
                                           0.22238103445337443f, 0.10122853629037706f};
 
-// log Phi(a); for a <= 0 through the scaled complement erfcx (no underflow).
-static __device__ __noinline__ float log_ndtr(float a) {
-  if (a > 0.0f) return log1pf(-0.5f * erfcf(a * kSqrtHalf));
-  return logf(0.5f * erfcxf(-a * kSqrtHalf)) - 0.5f * a * a;
+// (log Phi(a), g(a)) from one scaled complement E = erfcx(|a|/sqrt 2)/2 =
+// Phi(-|a|) e^{a^2/2}: for a <= 0, log Phi(a) = log E - a^2/2 (no underflow); for
+// a > 0, log Phi(a) = log(1 - E e^{-a^2/2}).  Both branches are computed and one is
+// selected, so that lanes with different arguments do not diverge.
+__device__ __forceinline__ float2 log_ndtr_g(float a) {
+  const float E = 0.5f * erfcxf(fabsf(a) * kSqrtHalf);
+  const float h = 0.5f * a * a;
+  const float lneg = logf(E);                  // log Phi(-|a|) + a^2/2
+  const float lpos = log1pf(-E * expf(-h));    // log Phi(|a|)
+  return (a <= 0.0f) ? make_float2(lneg - h, lneg) : make_float2(lpos, lpos + h);
 }
+
+// log Phi(a).
+static __device__ SDV_HELPER float log_ndtr(float a) { return log_ndtr_g(a).x; }
 
 // g(a) = log Phi(a) + a^2/2 (moderate for a <= 0).
-static __device__ __noinline__ float gfun(float a) {
-  if (a <= 0.0f) return logf(0.5f * erfcxf(-a * kSqrtHalf));
-  return log_ndtr(a) + 0.5f * a * a;
-}
+static __device__ SDV_HELPER float gfun(float a) { return log_ndtr_g(a).y; }
 
-// g'(s) = lambda(s) + s > 0.  The continued fraction is evaluated bottom-up with a
-// fast reciprocal: each level adds n/acc << x to x, so the reciprocal's few-ulp
-// error is damped by the levels above; only the final division is exact.  Deeper
-// levels are needed only near the switch point (16 levels give ~5e-10 at x = 4,
-// 8 levels ~4e-10 at x = 8).
-__device__ __forceinline__ float gprime(float s) {
-  if (s < -4.0f) {
-    const float x = -s;
-    float acc = x;
-    if (x < 8.0f) {
+// g'(s) = lambda(s) + s > 0 in its two forms.  For s < -4 (x = -s) Laplace's
+// continued fraction for the Mills ratio with its first term cancelled,
+// lambda(s) + s = 1/(x + 2/(x + 3/(x + ... 16/x))), written as 1/(x c) with
+// c = 1 + 2u/(1 + 3u/(1 + ... 16u)), u = 1/x^2 <= 1/16, and c evaluated by the
+// forward three-term recurrence (fused multiply-adds on positive terms, one
+// division); 15 levels give ~5e-10 relative at x = 4 and less beyond.  Elsewhere
+// sqrt(2/pi)/erfcx(-s/sqrt 2) + s, which tends to s for large s as erfcx overflows.
+__device__ __forceinline__ float gprime_cf(float s) {
+  const float x = fmaxf(-s, 4.0f);
+  const float u = 1.0f / (x * x);
+  float a0 = 1.0f, a1 = 1.0f, b0 = 0.0f, b1 = 1.0f;  // A_{n-2}, A_{n-1}, B_{n-2}, B_{n-1}
 #pragma unroll
-      for (int n = 16; n >= 9; --n) acc = x + __fdividef((float)n, acc);
-    }
-#pragma unroll
-    for (int n = 8; n >= 2; --n) acc = x + __fdividef((float)n, acc);
-    return 1.0f / acc;
+  for (int n = 2; n <= 16; ++n) {
+    const float an = (float)n * u;
+    const float a2 = fmaf(an, a0, a1), b2 = fmaf(an, b0, b1);
+    a0 = a1; a1 = a2; b0 = b1; b1 = b2;
   }
-  // lambda(s) = phi(s)/Phi(s) = sqrt(2/pi) / erfcx(-s/sqrt 2); beyond s = 9 it is < 1e-18
-  if (s > 9.0f) return s;
+  return b1 / (x * a1);
+}
+__device__ __forceinline__ float gprime_ex(float s) {
   return 0.79788456080286536f / erfcxf(-s * kSqrtHalf) + s;
 }
 
@@ -146,31 +169,65 @@ __device__ __forceinline__ float gprime(float s) {
 // difference of two g values is accurate to a few 1e-7 absolute (|g| <= ~3 for
 // arguments above -8); it is replaced by 8-point Gauss-Legendre quadrature of g'
 // where the difference itself is small: short intervals and the deep left tail
-// (g' ~ 1/|s| there).
-static __device__ __noinline__ float gdiff(float hi, float h) {
-  const bool careful = (h < 0.5f) || (hi < -2.0f);
-  if (careful && h <= fmaxf(2.0f, 0.5f * fabsf(hi))) {
+// (g' ~ 1/|s| there).  The choice of form (and, inside the quadrature, of the
+// form of g') is voted over the converged lanes, and every form that some lane
+// needs is evaluated by all of them as straight-line code (the eight nodes
+// interleave); lanes with different arguments therefore never diverge.
+static __device__ SDV_HELPER float gdiff(float hi, float h) {
+  const unsigned act = __activemask();
+  const bool careful = ((h < 0.5f) || (hi < -2.0f)) && (h <= fmaxf(2.0f, 0.5f * fabsf(hi)));
+  float quad = 0.0f, direct = 0.0f;
+  if (__any_sync(act, careful)) {
     const float r = 0.5f * h, m = hi - r;
+    float sv[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      sv[2 * i] = m + r * kGLx[i];
+      sv[2 * i + 1] = m - r * kGLx[i];
+    }
+    // nodes lie in [hi - h, hi]
+    const bool need_cf = __any_sync(act, careful && hi - h < -4.0f);
+    const bool need_ex = __any_sync(act, careful && hi >= -4.0f);
+    float gp[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) gp[i] = 0.0f;
+    if (need_ex) {
+#pragma unroll kGLUnroll
+      for (int i = 0; i < 8; ++i) gp[i] = gprime_ex(sv[i]);
+    }
+    if (need_cf) {
+#pragma unroll kGLUnroll
+      for (int i = 0; i < 8; ++i) {
+        const float cf = gprime_cf(sv[i]);
+        gp[i] = (sv[i] < -4.0f) ? cf : gp[i];
+      }
+    }
     float acc = 0.0f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      acc += kGLw[i] * (gprime(m + r * kGLx[i]) + gprime(m - r * kGLx[i]));
-    return r * acc;
+    for (int i = 0; i < 4; ++i) acc += kGLw[i] * (gp[2 * i] + gp[2 * i + 1]);
+    quad = r * acc;
   }
-  const float lo = hi - h;
-  if (hi <= 0.0f) return gfun(hi) - gfun(lo);
-  return (log_ndtr(hi) - log_ndtr(lo)) + h * (hi - 0.5f * h);
+  if (__any_sync(act, !careful)) {
+    const float lo = hi - h;
+    const float2 ph = log_ndtr_g(hi), pl = log_ndtr_g(lo);
+    direct = (hi <= 0.0f) ? ph.y - pl.y : (ph.x - pl.x) + h * (hi - 0.5f * h);
+  }
+  return careful ? quad : direct;
 }
 
-// log(1 - e^x), x <= 0.
+// log(1 - e^x), x <= 0 (both forms evaluated, one selected).
 __device__ __forceinline__ float log1mexp(float x) {
   x = fminf(x, 0.0f);
-  return (x > -kLn2) ? logf(-expm1f(x)) : log1pf(-expf(x));
+  const float near0 = logf(-expm1f(x));
+  const float far = log1pf(-expf(x));
+  return (x > -kLn2) ? near0 : far;
 }
 
-// log(e^y - 1), y >= 0.
+// log(e^y - 1), y >= 0 (both forms evaluated, one selected).
 __device__ __forceinline__ float logexpm1(float y) {
-  return (y > 15.0f) ? y + log1pf(-expf(-y)) : logf(expm1f(y));
+  const float big = y + log1pf(-expf(-y));
+  const float small = logf(expm1f(fminf(y, 15.0f)));
+  return (y > 15.0f) ? big : small;
 }
 
 __device__ __forceinline__ float logaddexp(float a, float b) {
@@ -180,56 +237,74 @@ __device__ __forceinline__ float logaddexp(float a, float b) {
 }
 
 // log(Phi(b) - Phi(a)) for a < b.
-static __device__ __noinline__ float log_ndtr_interval(float a, float b) {
+static __device__ SDV_HELPER float log_ndtr_interval(float a, float b) {
   if (b <= 0.0f) return log_ndtr(b) + log1mexp(log_ndtr(a) - log_ndtr(b));
   if (a >= 0.0f) return log_ndtr(-a) + log1mexp(log_ndtr(-b) - log_ndtr(-a));
   return log1pf(-(expf(log_ndtr(a)) + expf(log_ndtr(-b))));
 }
 
 // ---------------------------------------------------------------- block verification
-// log h_j, h_j = v_j / (v_j + 1 - alpha_j), from log alpha_j (<= 0) and |Delta_{j+1}|.
-// Limits: alpha_j = 1 -> h = 1; alpha_j = 0 or |Delta_{j+1}| = 0 (alpha_j < 1) -> h = 0.
-static __device__ __noinline__ float block_log_h(float la, float Dn) {
+// log h_j, h_j = v_j / (v_j + 1 - alpha_j), from log alpha_j (<= 0), |Delta_{j+1}| and
+// log v_j, the residual mass of step j + 1 at alpha_j (usample_setup(|Delta_{j+1}|,
+// log alpha_j).lv).  Limits: alpha_j = 1 -> h = 1; alpha_j = 0 or |Delta_{j+1}| = 0
+// (alpha_j < 1) -> h = 0.
+__device__ __forceinline__ float block_log_h(float la, float Dn, float lv) {
   if (isnan(la) || isnan(Dn)) return -INFINITY;
   if (!(la < 0.0f)) return 0.0f;
   if (la == -INFINITY || !(Dn > 0.0f)) return -INFINITY;
+  return lv - logaddexp(lv, log1mexp(la));
+}
+
+// log h_j from log alpha_j and |Delta_{j+1}| alone (evaluates log v_j).
+static __device__ SDV_HELPER float block_log_h(float la, float Dn) {
+  if (isnan(la) || isnan(Dn) || !(la < 0.0f) || la == -INFINITY || !(Dn > 0.0f))
+    return block_log_h(la, Dn, 0.0f);  // the limits, which do not read log v
   const float ap = la / Dn + 0.5f * Dn;
   const float x0 = -gdiff(ap, Dn);              // log(Phi(a-) / (alpha Phi(a+)))
   const float lv = la + log_ndtr(ap) + log1mexp(x0);
-  const float l1ma = log1mexp(la);              // log(1 - alpha)
-  return lv - logaddexp(lv, l1ma);
+  return block_log_h(la, Dn, lv);
 }
 
 // ---------------------------------------------------------------- residual U-sampler
 struct UParams {
   float D, la, ap, am;
-  float lv;   // log v
-  float lvn;  // log v - log phi(a-)
+  float lv;      // log v
+  float lvn;     // log v - log phi(a-)
+  float lnd_ap;  // log Phi(a+)
+  float g_ap;    // g(a+)
+  float l1mx0;   // log(1 - e^{x0}) = log(v / (alpha Phi(a+)))
 };
 
-static __device__ __noinline__ UParams usample_setup(float D, float la) {
+static __device__ SDV_HELPER UParams usample_setup(float D, float la) {
   UParams P;
   P.D = D;
   P.la = la;
   P.ap = la / D + 0.5f * D;
   P.am = P.ap - D;
   const float x0 = -gdiff(P.ap, D);
-  P.lv = la + log_ndtr(P.ap) + log1mexp(x0);
+  const float2 lg = log_ndtr_g(P.ap);
+  P.lnd_ap = lg.x;
+  P.g_ap = lg.y;
+  P.l1mx0 = log1mexp(x0);
+  P.lv = la + P.lnd_ap + P.l1mx0;
   P.lvn = gfun(P.am) + kHalfLog2Pi + logexpm1(-x0);
   return P;
 }
 
-// log Psi(a+ - t), t > 0.
-static __device__ __noinline__ float usample_log_psi(float t, const UParams& P) {
+// log Psi(a+ - t), t > 0, as [log Phi(u) - log Phi(a+)] + log(1 - e^x) - log(1 - e^{x0}),
+// u = a+ - t: Psi(u) = alpha Phi(u) (1 - e^x) / v and v = alpha Phi(a+) (1 - e^{x0}).
+// The first bracket is g(u) - g(a+) + t (a+ + u)/2 for a+ <= 0 (no term larger than
+// the result grows with |a+|) and a plain difference of log Phi otherwise.
+static __device__ SDV_HELPER float usample_log_psi(float t, const UParams& P) {
   const float u = P.ap - t;
   const float x = -gdiff(u, P.D) - P.D * t;     // log(Phi(u - D) / (alpha Phi(u)))
-  if (u < 0.0f)
-    return gfun(u) + log1mexp(x) - P.lvn + kHalfLog2Pi + 0.5f * t * (P.ap + u);
-  return P.la + log_ndtr(u) + log1mexp(x) - P.lv;
+  const float2 lg = log_ndtr_g(u);
+  const float dl = (P.ap <= 0.0f) ? (lg.y - P.g_ap) + 0.5f * t * (P.ap + u) : lg.x - P.lnd_ap;
+  return dl + log1mexp(x) - P.l1mx0;
 }
 
 // log(1 - Psi(a+ - t)), t > 0.
-static __device__ __noinline__ float usample_log_1mpsi(float t, const UParams& P) {
+static __device__ SDV_HELPER float usample_log_1mpsi(float t, const UParams& P) {
   if (P.D * t <= 1.0f && -P.am * t <= 4.0f) {
     const float r = 0.5f * t;
     float acc = 0.0f;
@@ -316,6 +391,70 @@ __device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits
     hi = sm->t[1];
     ghi = sm->g[1];
     __syncthreads();
+  }
+  // Newton step from the closer end
+  const bool from_lo = isfinite(glo) && (-glo < ghi);
+  const float te = from_lo ? lo : hi, ge = from_lo ? glo : ghi;
+  const float lpsi = P.am * te - 0.5f * te * te + logexpm1(P.D * te) - P.lvn;
+  const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
+  const float dg = expf(lpsi - lden);
+  // Return u directly: u_e = fl(a+ - t_e) is the point the evaluator used, so adding
+  // the Newton correction keeps U's rounding relative to |U| rather than to |a+|.
+  const float ue = P.ap - te;
+  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
+  step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
+  return ue + step;
+}
+
+// U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32, by one converged warp: every lane
+// passes the same P (from usample_setup) and wbits and returns U.  Work in
+// t = a+ - u (Psi decreases in t) with the gap g(t) = log w - log Psi (lower half
+// of w) or log(1 - Psi) - log(1 - w) (upper half), increasing in t and >= 0
+// exactly when Psi(a+ - t) <= w:
+//  1. bracket: the 32 candidates t_k = s0 2^(k - 8) (the paper's doubling of the
+//     bracket, all steps at once), s0 = 1/max(1, |a-|) the residual's scale;
+//  2. kURounds rounds of 32-way multisection (each shrinks the bracket 32-fold);
+//  3. one Newton step from the bracket end with the smaller |g|, clamped to the
+//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form,
+//     log psi(a+ - t) = a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)).
+constexpr int kURounds = 3;
+
+__device__ __forceinline__ float usample_warp(const UParams& P, uint32_t wbits, uint32_t* status) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const bool upper = wbits >= 0x80000000u;
+  const float target = upper ? logf(((float)(0xFFFFFFFFu - wbits) + 0.5f) * 0x1p-32f)
+                             : logf(((float)wbits + 0.5f) * 0x1p-32f);
+  auto gap = [&](float t) -> float {
+    if (upper) return usample_log_1mpsi(t, P) - target;
+    return target - usample_log_psi(t, P);
+  };
+  const float s0 = 1.0f / fmaxf(1.0f, fabsf(P.am));
+  const float tk = s0 * exp2f((float)lane - 8.0f);
+  const float gk = gap(tk);
+  unsigned m = __ballot_sync(FULL, gk >= 0.0f);
+  if (m == 0u) {
+    *status |= 4u;  // SDV_STATUS_USAMPLE_RANGE
+    return P.ap - s0 * exp2f(24.0f);
+  }
+  int f = __ffs(m) - 1;
+  float hi = __shfl_sync(FULL, tk, f), ghi = __shfl_sync(FULL, gk, f);
+  const float tp = __shfl_sync(FULL, tk, (f + 31) & 31), gp = __shfl_sync(FULL, gk, (f + 31) & 31);
+  float lo = (f == 0) ? 0.0f : tp;
+  float glo = (f == 0) ? -INFINITY : gp;
+#pragma unroll 1
+  for (int r = 0; r < kURounds; ++r) {
+    const float h = (hi - lo) * (1.0f / 32.0f);
+    const float t = (lane < 31) ? lo + (float)(lane + 1) * h : hi;
+    const float gt0 = gap(t);                 // every lane evaluates (converged votes)
+    const float gt = (lane < 31) ? gt0 : ghi;  // the upper end keeps its known value
+    m = __ballot_sync(FULL, gt >= 0.0f);       // lane 31 always votes true
+    f = __ffs(m) - 1;
+    const float nt = __shfl_sync(FULL, t, f), ng = __shfl_sync(FULL, gt, f);
+    const float pt = __shfl_sync(FULL, t, (f + 31) & 31), pg = __shfl_sync(FULL, gt, (f + 31) & 31);
+    if (f > 0) { lo = pt; glo = pg; }
+    hi = nt;
+    ghi = ng;
   }
   // Newton step from the closer end
   const bool from_lo = isfinite(glo) && (-glo < ghi);

@@ -219,6 +219,7 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
         // partials written by other CTAs of this grid: read through L2
         const float2* p = A.part + ((int64_t)b * L + j) * A.C;
         float a1 = 0.f, a2 = 0.f;
+#pragma unroll 16
         for (int c = 0; c < A.C; ++c) {
           const float2 t = __ldcg(p + c);
           a1 += t.x;

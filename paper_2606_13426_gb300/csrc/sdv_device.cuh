@@ -330,7 +330,8 @@ struct USampleScratch {
 };
 
 // U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32, by all NT threads of a CTA (NT a
-// multiple of 32, <= 1024) with the same arguments; every thread returns U.
+// multiple of 32, <= 1024) with the same arguments (P from usample_setup); every
+// thread returns U.
 // Work in t = a+ - u (Psi decreases in t) with the gap g(t) = log w - log Psi
 // (lower half of w) or log(1 - Psi) - log(1 - w) (upper half), increasing in t
 // and >= 0 exactly when Psi(a+ - t) <= w:
@@ -342,11 +343,10 @@ struct USampleScratch {
 //     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form,
 //     log psi(a+ - t) = a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)).
 template <int NT>
-__device__ __forceinline__ float usample_block(float D, float la, uint32_t wbits,
-                                               uint32_t* status, USampleScratch* sm) {
+__device__ __forceinline__ float usample_block(const UParams& P, uint32_t wbits, uint32_t* status,
+                                               USampleScratch* sm) {
   const unsigned FULL = 0xffffffffu;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const UParams P = usample_setup(D, la);
   const bool upper = wbits >= 0x80000000u;
   const float target = upper ? logf(((float)(0xFFFFFFFFu - wbits) + 0.5f) * 0x1p-32f)
                              : logf(((float)wbits + 0.5f) * 0x1p-32f);

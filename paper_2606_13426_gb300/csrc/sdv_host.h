@@ -11,6 +11,9 @@ namespace sdv {
 // Fused verify kernel: threads per CTA and 16-byte vectors per thread per tensor per sweep.
 constexpr int kK1Threads = 256;
 constexpr int kK1Vpt = 4;
+// Resident CTAs per SM the fused kernel is built for (its register budget): the
+// chain-finishing code needs more than the streaming loop.
+constexpr int kK1MinBlocks = 3;
 // Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;
 // Long-row residual kernels: threads per CTA and elements of the rejected row per CTA.
@@ -18,7 +21,7 @@ constexpr int kK4Threads = 256;
 constexpr int kK4Chunk = 4096;
 // Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
 // finishes the chain inside the fused kernel; longer rows by k_resid_dot/_write.
-constexpr int64_t kFusedMaxGroups = 4096;
+constexpr int64_t kFusedMaxGroups = 1024;
 
 enum : int32_t {
   kKindInactive = 0,

@@ -187,10 +187,34 @@ __device__ __forceinline__ ChainState inactive_state() {
   return cs;
 }
 
-// For chain b: ell_j, |Delta_j| (from the tile partials, or given), coins, the
-// acceptance rule, and the residual 1-D draw.  Called by a full warp; every lane
-// returns the chain's ChainState.  Writes the per-chain outputs of ScanArgs.
-__device__ ChainState scan_warp(const ScanArgs& A, int b) {
+struct ScanOut {
+  ChainState cs;
+  UParams P;   // residual parameters of row tau - 1 (block mode, cs.kind == kKindResid)
+  bool have_P;
+};
+
+__device__ __forceinline__ UParams shfl_params(const UParams& P, int src) {
+  const unsigned FULL = 0xffffffffu;
+  UParams R;
+  R.D = __shfl_sync(FULL, P.D, src);
+  R.la = __shfl_sync(FULL, P.la, src);
+  R.ap = __shfl_sync(FULL, P.ap, src);
+  R.am = __shfl_sync(FULL, P.am, src);
+  R.lv = __shfl_sync(FULL, P.lv, src);
+  R.lvn = __shfl_sync(FULL, P.lvn, src);
+  R.lnd_ap = __shfl_sync(FULL, P.lnd_ap, src);
+  R.g_ap = __shfl_sync(FULL, P.g_ap, src);
+  R.l1mx0 = __shfl_sync(FULL, P.l1mx0, src);
+  return R;
+}
+
+// For chain b: ell_j, |Delta_j| (from the tile partials, or given), coins and the
+// acceptance rule.  In block mode every candidate residual row j (lane j & 31 of
+// segment j >> 5) also gets the U-sampler setup at (|Delta_j|, log alpha_{j-1})
+// (log alpha_{-1} = 0), whose log v is the residual mass that h_{j-1} needs: the
+// scan evaluates it once for both.  Called by a full warp; every lane returns the
+// result.  Writes the per-chain outputs of ScanArgs except status and aux.
+__device__ ScanOut scan_warp(const ScanArgs& A, int b) {
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int L = A.L;
@@ -205,7 +229,10 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
       for (int j = lane; j < L; j += 32) A.ell_out[(int64_t)b * L + j] = 0.f;
     if (A.dn_out)
       for (int j = lane; j < L; j += 32) A.dn_out[(int64_t)b * L + j] = 0.f;
-    return inactive_state();
+    ScanOut o;
+    o.cs = inactive_state();
+    o.have_P = false;
+    return o;
   }
   const int nseg = (L + 31) >> 5;
   float ell[2], dn[2], S1[2], S2[2], sg[2];
@@ -242,7 +269,12 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
     }
   }
   const bool any_bad = __any_sync(FULL, bad);
-  if (A.ratios_only) return inactive_state();
+  ScanOut out;
+  out.have_P = false;
+  if (A.ratios_only) {
+    out.cs = inactive_state();
+    return out;
+  }
 
   // coins: eta_j from Philox (b, j, 0, 0), word 0, compared in log space
   float leta[2];
@@ -269,24 +301,53 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
     tau = fm[0] ? __ffs(fm[0]) : (fm[1] ? 32 + __ffs(fm[1]) : g + 1);
   } else {
     // block verification: log alpha_j = min{0, log alpha_{j-1} + ell_j}, evaluated in
-    // step order (lane j & 31 of segment j >> 5 keeps log alpha_j), so that a clamp to
-    // alpha = 1 is exact exactly when the recursion reaches it
+    // step order by every lane on all tempered ell (gathered with independent
+    // shuffles), lane j & 31 of segment j >> 5 keeping log alpha_j, so that a clamp
+    // to alpha = 1 is exact exactly when the recursion reaches it
     float la[2] = {0.f, 0.f};
     float run = 0.f;
-#pragma unroll 4
-    for (int j = 0; j < g; ++j) {
-      const float e0 = __shfl_sync(FULL, ellw[0], j & 31);
-      const float e1 = __shfl_sync(FULL, ellw[1], j & 31);
-      run = fminf(0.f, run + (j < 32 ? e0 : e1));
-      if (lane == (j & 31)) {
-        if (j < 32) la[0] = run;
-        else la[1] = run;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float e = __shfl_sync(FULL, ellw[0], k);
+      const float nr = fminf(0.f, run + e);
+      run = (k < g) ? nr : run;
+      la[0] = (k == lane) ? run : la[0];
+    }
+    if (nseg > 1) {  // warp-uniform
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const float e = __shfl_sync(FULL, ellw[1], k);
+        const float nr = fminf(0.f, run + e);
+        run = (32 + k < g) ? nr : run;
+        la[1] = (k == lane) ? run : la[1];
       }
     }
-    // h_j (0-based j) uses |Delta| of step j + 1 (the paper's D_{j+1} in 1-based steps)
-    const float dn_next0 = __shfl_down_sync(FULL, dn[0], 1);
-    const float dn_first1 = __shfl_sync(FULL, dn[1], 0);
-    const float dn_next1 = __shfl_down_sync(FULL, dn[1], 1);
+    // log alpha_{j-1} of each candidate residual row, and its U-sampler setup
+    float lap[2];
+    {
+      const float up0 = __shfl_up_sync(FULL, la[0], 1);
+      const float last0 = __shfl_sync(FULL, la[0], 31);
+      const float up1 = __shfl_up_sync(FULL, la[1], 1);
+      lap[0] = (lane == 0) ? 0.f : up0;
+      lap[1] = (lane == 0) ? last0 : up1;
+    }
+    UParams Pq[2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      if (q < nseg) {  // warp-uniform
+        const bool ok = (dn[q] > 0.f) && isfinite(dn[q]) && isfinite(lap[q]);
+        Pq[q] = usample_setup(ok ? dn[q] : 1.f, ok ? fminf(lap[q], 0.f) : -1.f);
+      } else {
+        Pq[q] = UParams{};
+      }
+    }
+    // h_j (0-based j) uses |Delta| and log v of step j + 1 (the paper's D_{j+1})
+    const float dnx0 = __shfl_down_sync(FULL, dn[0], 1);
+    const float dnx1 = __shfl_down_sync(FULL, dn[1], 1);
+    const float dnf1 = __shfl_sync(FULL, dn[1], 0);
+    const float lvx0 = __shfl_down_sync(FULL, Pq[0].lv, 1);
+    const float lvx1 = __shfl_down_sync(FULL, Pq[1].lv, 1);
+    const float lvf1 = __shfl_sync(FULL, Pq[1].lv, 0);
     unsigned sm[2];
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
@@ -297,8 +358,9 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
         if (j == g - 1) {
           lh = la[q];  // h_gamma = alpha_gamma
         } else {
-          const float Dn = (q == 0) ? (lane == 31 ? dn_first1 : dn_next0) : dn_next1;
-          lh = block_log_h(la[q], Dn);
+          const float Dn = (q == 0) ? (lane == 31 ? dnf1 : dnx0) : dnx1;
+          const float lv = (q == 0) ? (lane == 31 ? lvf1 : lvx0) : lvx1;
+          lh = block_log_h(la[q], Dn, lv);
         }
         succ = leta[q] < lh;
       }
@@ -313,6 +375,13 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
       const float v0 = __shfl_sync(FULL, la[0], k & 31);
       const float v1 = __shfl_sync(FULL, la[1], k & 31);
       la_res = (k < 32) ? v0 : v1;
+    }
+    if (tau <= g) {  // residual parameters of row tau - 1
+      const int rr = tau - 1;
+      const UParams P0 = shfl_params(Pq[0], rr & 31);
+      const UParams P1 = shfl_params(Pq[1], rr & 31);
+      out.P = (rr >> 5) ? P1 : P0;
+      out.have_P = true;
     }
   }
 
@@ -342,7 +411,7 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
     if (A.tau_out) A.tau_out[b] = tau;
     if (A.la_res_out) A.la_res_out[b] = la_res;
   }
-  ChainState cs;
+  ChainState& cs = out.cs;
   cs.tau = tau;
   cs.row = resid ? rrow : g - 1;
   cs.U = NAN;
@@ -354,18 +423,19 @@ __device__ ChainState scan_warp(const ScanArgs& A, int b) {
   cs.status = status;
   cs.kind = kind;
   cs.pad[0] = cs.pad[1] = 0;
-  return cs;
+  return out;
 }
 
 // Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch), then
 // the outputs that depend on it: status bits and (U, log alpha_res, |Delta_tau|, sigma_tau).
 template <int NT>
 __device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, ChainState& cs,
-                                                  USampleScratch* us) {
+                                                  const UParams* P, USampleScratch* us) {
   if (cs.kind == kKindResid && A.draw_u) {
     const uint32_t wbits = philox_block(A.seed, (uint32_t)b, 0u, kStreamUSample, 0u).x;
     uint32_t st = cs.status;
-    cs.U = usample_block<NT>(cs.dnorm, fminf(cs.la_res, 0.f), wbits, &st, us);
+    const UParams Q = P ? *P : usample_setup(cs.dnorm, fminf(cs.la_res, 0.f));
+    cs.U = usample_block<NT>(Q, wbits, &st, us);
     cs.status = st;
   }
   if (threadIdx.x == 0 && cs.kind != kKindInactive) {
@@ -384,7 +454,10 @@ __device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, Chai
 // Writes y[b, :] for chain state cs with the whole CTA (blockDim.x threads, a
 // multiple of 32).  Decomposition: pass A reduces delta^T G, pass B writes
 // m^q + sigma (G + e (U - e^T G)), drawing G again (same Philox counters) rather
-// than holding the row on chip.
+// than holding the row on chip.  Each thread handles kResidUnroll groups of four
+// elements per sweep, loads and Philox blocks of all of them issued together.
+constexpr int kResidUnroll = 1;
+
 template <typename T, bool VEC4>
 __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
                              const T* __restrict__ mp, const T* __restrict__ mq_bonus,
@@ -392,21 +465,29 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
                              uint64_t seed, int b, const ChainState& cs, T* __restrict__ y,
                              float2* red, float* bcast) {
   if (cs.kind == kKindInactive) return;
+  constexpr int RU = kResidUnroll;
   const int nt = blockDim.x;
   const int64_t ng = (d + 3) / 4;
   const int64_t rbase = ((int64_t)b * L + cs.row) * d;
   const int64_t ybase = (int64_t)b * d;
+  // groups past the row end load zeros (load4 guards each element) and store nothing
   if (cs.kind == kKindResid) {
     float sp = 0.f;
-    for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
-      float fq[4], fp[4];
-      load4<T, VEC4>(mq + rbase, 4 * gi, d, fq);
-      load4<T, VEC4>(mp + rbase, 4 * gi, d, fp);
-      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-      sp = fmaf(fp[0] - fq[0], G.x, sp);  // tail lanes load 0 and contribute 0
-      sp = fmaf(fp[1] - fq[1], G.y, sp);
-      sp = fmaf(fp[2] - fq[2], G.z, sp);
-      sp = fmaf(fp[3] - fq[3], G.w, sp);
+    for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
+      float fq[RU][4], fp[RU][4];
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
+        load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)(g0 + (int64_t)u * nt), kStreamResid, 0u);
+        sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
+        sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
+        sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
+        sp = fmaf(fp[u][3] - fq[u][3], G.w, sp);
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) sp += __shfl_xor_sync(0xffffffffu, sp, o);
@@ -420,46 +501,64 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
     }
     __syncthreads();
     const float coef = *bcast;
-    for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
-      float fq[4], fp[4], out[4];
-      load4<T, VEC4>(mq + rbase, 4 * gi, d, fq);
-      load4<T, VEC4>(mp + rbase, 4 * gi, d, fp);
-      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-      const float g4[4] = {G.x, G.y, G.z, G.w};
+    for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
+      float fq[RU][4], fp[RU][4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k)
-        out[k] = fq[k] + cs.sigma * fmaf((fp[k] - fq[k]) * cs.inv_norm, coef, g4[k]);
-      store4<T, VEC4>(y + ybase, 4 * gi, d, out);
+      for (int u = 0; u < RU; ++u) {
+        load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
+        load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        const int64_t gi = g0 + (int64_t)u * nt;
+        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+        const float g4[4] = {G.x, G.y, G.z, G.w};
+        float out[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          out[k] = fq[u][k] + cs.sigma * fmaf((fp[u][k] - fq[u][k]) * cs.inv_norm, coef, g4[k]);
+        if (gi < ng) store4<T, VEC4>(y + ybase, 4 * gi, d, out);
+      }
     }
     return;
   }
-  for (int64_t gi = threadIdx.x; gi < ng; gi += nt) {
-    const int64_t i = 4 * gi;
-    float out[4];
-    if (cs.kind == kKindReflect) {
-      float fx[4], fq[4], fp[4];
-      load4<T, VEC4>(x + rbase, i, d, fx);
-      load4<T, VEC4>(mq + rbase, i, d, fq);
-      load4<T, VEC4>(mp + rbase, i, d, fp);
+  const bool bonus = cs.kind == kKindBonus;
+  const bool draw = bonus || cs.kind == kKindZeroDelta;
+  const float sgm = bonus ? sigma_bonus[b] : cs.sigma;
+  for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
+    float a[RU][4], q[RU][4], p[RU][4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) out[k] = fx[k] - (fp[k] - fq[k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
-    } else if (cs.kind == kKindZeroDelta) {
-      float fq[4];
-      load4<T, VEC4>(mq + rbase, i, d, fq);
-      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-      out[0] = fq[0] + cs.sigma * G.x; out[1] = fq[1] + cs.sigma * G.y;
-      out[2] = fq[2] + cs.sigma * G.z; out[3] = fq[3] + cs.sigma * G.w;
-    } else if (cs.kind == kKindBonus) {
-      float fb[4];
-      load4<T, VEC4>(mq_bonus + ybase, i, d, fb);
-      const float sb = sigma_bonus[b];
-      const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamBonus, 0u);
-      out[0] = fb[0] + sb * G.x; out[1] = fb[1] + sb * G.y;
-      out[2] = fb[2] + sb * G.z; out[3] = fb[3] + sb * G.w;
-    } else {  // copy the last accepted draft
-      load4<T, VEC4>(x + rbase, i, d, out);
+    for (int u = 0; u < RU; ++u) {
+      const int64_t i = 4 * (g0 + (int64_t)u * nt);
+      if (cs.kind == kKindReflect) {
+        load4<T, VEC4>(x + rbase, i, d, a[u]);
+        load4<T, VEC4>(mq + rbase, i, d, q[u]);
+        load4<T, VEC4>(mp + rbase, i, d, p[u]);
+      } else if (cs.kind == kKindZeroDelta) {
+        load4<T, VEC4>(mq + rbase, i, d, a[u]);
+      } else if (bonus) {
+        load4<T, VEC4>(mq_bonus + ybase, i, d, a[u]);
+      } else {  // copy the last accepted draft
+        load4<T, VEC4>(x + rbase, i, d, a[u]);
+      }
     }
-    store4<T, VEC4>(y + ybase, i, d, out);
+#pragma unroll
+    for (int u = 0; u < RU; ++u) {
+      const int64_t gi = g0 + (int64_t)u * nt;
+      float out[4];
+      if (cs.kind == kKindReflect) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) out[k] = a[u][k] - (p[u][k] - q[u][k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
+      } else if (draw) {
+        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, bonus ? kStreamBonus : kStreamResid, 0u);
+        out[0] = a[u][0] + sgm * G.x; out[1] = a[u][1] + sgm * G.y;
+        out[2] = a[u][2] + sgm * G.z; out[3] = a[u][3] + sgm * G.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) out[k] = a[u][k];
+      }
+      if (gi < ng) store4<T, VEC4>(y + ybase, 4 * gi, d, out);
+    }
   }
 }
 
@@ -481,11 +580,13 @@ struct VerifyArgs {
 
 // RESID: 1 = this kernel writes y; 0 = it leaves the chain state for k_resid_*.
 template <typename T, bool VEC, int VPT, bool VEC4, int RESID>
-__global__ void __launch_bounds__(kK1Threads, 4) k_verify(VerifyArgs A) {
+__global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs A) {
   __shared__ float2 red[kK1Threads / 32];
   __shared__ int last_s;
   __shared__ float bcast;
   __shared__ ChainState cs_s;
+  __shared__ UParams P_s;
+  __shared__ bool haveP_s;
   __shared__ USampleScratch us;
   const int L = A.S.L;
   const int C = A.S.C;
@@ -500,7 +601,7 @@ __global__ void __launch_bounds__(kK1Threads, 4) k_verify(VerifyArgs A) {
   if (g == 0) {
     // inactive chain: tile (b, 0, 0) writes its outputs, nothing is streamed
     if (j == 0 && c == 0 && threadIdx.x < 32) {
-      const ChainState cs = scan_warp(A.S, b);
+      const ChainState cs = scan_warp(A.S, b).cs;
       if (threadIdx.x == 0 && RESID == 0) A.state[b] = cs;
     }
     return;
@@ -520,13 +621,17 @@ __global__ void __launch_bounds__(kK1Threads, 4) k_verify(VerifyArgs A) {
   if (!last_s) return;
   __threadfence();  // acquire: every partial of chain b is visible
   if (threadIdx.x < 32) {
-    const ChainState cs = scan_warp(A.S, b);
-    if (threadIdx.x == 0) cs_s = cs;
+    const ScanOut so = scan_warp(A.S, b);
+    if (threadIdx.x == 0) {
+      cs_s = so.cs;
+      P_s = so.P;
+      haveP_s = so.have_P;
+    }
   }
   __syncthreads();
   if (A.S.ratios_only) return;
   ChainState cs = cs_s;
-  draw_u_and_report<kK1Threads>(A.S, b, cs, &us);
+  draw_u_and_report<kK1Threads>(A.S, b, cs, haveP_s ? &P_s : nullptr, &us);
   if (RESID == 0) {
     if (threadIdx.x == 0) A.state[b] = cs;
   } else {
@@ -539,7 +644,7 @@ __global__ void __launch_bounds__(kK1Threads, 4) k_verify(VerifyArgs A) {
 __global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
   const int b = blockIdx.x * (kK2Threads / 32) + (threadIdx.x >> 5);
   if (b >= A.B) return;  // warp-uniform
-  scan_warp(A, b);
+  (void)scan_warp(A, b);
 }
 
 // ---------------------------------------------------------------- long rows: K4a / K4b
@@ -643,7 +748,7 @@ k_usample(const float* __restrict__ D, const float* __restrict__ la, const uint3
     status = 1u;
   } else {
     l = fminf(l, 0.f);
-    u = usample_block<kK1Threads>(Dn, l, w[i], &status, &us);
+    u = usample_block<kK1Threads>(usample_setup(Dn, l), w[i], &status, &us);
   }
   if (threadIdx.x == 0) {
     U[i] = u;

@@ -308,22 +308,29 @@ int sdv_em_sample(int B, int64_t d, const float *means, const float *log_weights
                   float t_floor, uint64_t seed, float *y_out, sdv_stream_t stream);
 
 /*
- * Profiling aid (not part of the method): when enabled, every later
- * sdv_verify / sdv_verify_ex call made on this host thread records four CUDA
- * events on its stream into a ring of `slots` entries: before the fused
- * verify kernel, after it, and (twice) after the separate residual kernels
- * used for rows longer than 16384 elements.  The records are ordinary stream
- * work, so they are captured into a CUDA graph like the kernels.  The events
- * are created here (host objects; no device memory).  slots = 0 disables
- * timing and destroys the events.
+ * Profiling aid (not part of the method): when enabled, sdv_verify /
+ * sdv_verify_ex calls made on this host thread record CUDA events on their
+ * stream into a ring of `slots` entries (one call in `every`, see
+ * sdv_timing_stride; every call by default): before the fused verify kernel,
+ * after it, and after the separate residual kernels used for rows longer than
+ * 4096 elements.  The records are ordinary stream work, so they are captured into
+ * a CUDA graph like the kernels (an event record costs a few microseconds of
+ * graph time, hence the stride).  The events are created here (host objects; no
+ * device memory).  slots = 0 disables timing and destroys the events.
  */
 int sdv_timing_enable(int slots);
+
+/*
+ * Records events for one call in `every` (every >= 1; the default 1 records
+ * every call) while timing is enabled.  SDV_EINVAL for every < 1.
+ */
+int sdv_timing_stride(int every);
 
 /*
  * Waits for the events of the last `n_calls` recorded calls (1 <= n_calls <=
  * slots) and writes their summed phase times in milliseconds:
  * ms3[0] the fused verify kernel (log-ratio pass, acceptance, U-draw and, for
- * rows up to 16384 elements, the residual write), ms3[1] the long-row residual
+ * rows up to 4096 elements, the residual write), ms3[1] the long-row residual
  * kernels (0 otherwise), ms3[2] reserved (0).  SDV_EINVAL if timing is off or
  * fewer calls were recorded.
  */

@@ -66,6 +66,7 @@ SIGNATURES = {
                              _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "sdv_em_sample": (_I, [_I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _P, _P]),
     "sdv_timing_enable": (_I, [_I]),
+    "sdv_timing_stride": (_I, [_I]),
     "sdv_timing_read": (_I, [_I, _P]),
 }
 
@@ -180,6 +181,10 @@ def sdv_normals(seed, B, d, stream_id, sub, out, stream):
 
 def sdv_timing_enable(slots):
     return _call("sdv_timing_enable", slots)
+
+
+def sdv_timing_stride(every):
+    return _call("sdv_timing_stride", every)
 
 
 def sdv_timing_read(n_calls):

@@ -33,9 +33,11 @@
 #ifndef SDV_HELPER
 #define SDV_HELPER __noinline__
 #endif
-// Unrolling of the quadrature nodes in gdiff (code size against node interleaving).
+// Unrolling of the quadrature nodes in gdiff.  The finishing path runs once per chain
+// from a cold instruction cache, where every 128-byte line of straight-line code costs a
+// fetch; a rolled node loop is far smaller than eight interleaved copies.
 #ifndef SDV_GL_UNROLL
-#define SDV_GL_UNROLL 8
+#define SDV_GL_UNROLL 1
 #endif
 namespace sdv {
 constexpr int kGLUnroll = SDV_GL_UNROLL;
@@ -113,6 +115,12 @@ __device__ __forceinline__ float4 normals4(uint64_t seed, uint32_t b, uint32_t b
   return make_float4(z01.x, z01.y, z23.x, z23.y);
 }
 
+// normals4 as one shared copy, for the residual paths that run once per chain.
+static __device__ SDV_HELPER float4 normals4_f(uint64_t seed, uint32_t b, uint32_t blk, uint32_t stream,
+                                               uint32_t sub) {
+  return normals4(seed, b, blk, stream, sub);
+}
+
 // ---------------------------------------------------------------- normal CDF helpers
 constexpr float kSqrtHalf = 0.70710678118654752f;
 constexpr float kHalfLog2Pi = 0.91893853320467274f;  // log(2 pi) / 2
@@ -124,12 +132,15 @@ static __constant__ float kGLx[4] = {0.18343464249564978f, 0.52553240991632899f,
 static __constant__ float kGLw[4] = {0.36268378337836166f, 0.31370664587788688f,
                                           0.22238103445337443f, 0.10122853629037706f};
 
+// One shared copy of the scaled complementary error function (see SDV_GL_UNROLL).
+static __device__ SDV_HELPER float erfcx_f(float x) { return erfcxf(x); }
+
 // (log Phi(a), g(a)) from one scaled complement E = erfcx(|a|/sqrt 2)/2 =
 // Phi(-|a|) e^{a^2/2}: for a <= 0, log Phi(a) = log E - a^2/2 (no underflow); for
 // a > 0, log Phi(a) = log(1 - E e^{-a^2/2}).  Both branches are computed and one is
 // selected, so that lanes with different arguments do not diverge.
 __device__ __forceinline__ float2 log_ndtr_g(float a) {
-  const float E = 0.5f * erfcxf(fabsf(a) * kSqrtHalf);
+  const float E = 0.5f * erfcx_f(fabsf(a) * kSqrtHalf);
   const float h = 0.5f * a * a;
   const float lneg = logf(E);                  // log Phi(-|a|) + a^2/2
   const float lpos = log1pf(-E * expf(-h));    // log Phi(|a|)
@@ -162,7 +173,7 @@ __device__ __forceinline__ float gprime_cf(float s) {
   return b1 / (x * a1);
 }
 __device__ __forceinline__ float gprime_ex(float s) {
-  return 0.79788456080286536f / erfcxf(-s * kSqrtHalf) + s;
+  return 0.79788456080286536f / erfcx_f(-s * kSqrtHalf) + s;
 }
 
 // g(hi) - g(hi - h) for h >= 0; the interval length is exactly h.  The direct

@@ -246,7 +246,7 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
         // partials written by other CTAs of this grid: read through L2
         const float2* p = A.part + ((int64_t)b * L + j) * A.C;
         float a1 = 0.f, a2 = 0.f;
-#pragma unroll 16
+#pragma unroll 4
         for (int c = 0; c < A.C; ++c) {
           const float2 t = __ldcg(p + c);
           a1 += t.x;
@@ -306,21 +306,12 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
     // to alpha = 1 is exact exactly when the recursion reaches it
     float la[2] = {0.f, 0.f};
     float run = 0.f;
-#pragma unroll
-    for (int k = 0; k < 32; ++k) {
-      const float e = __shfl_sync(FULL, ellw[0], k);
-      const float nr = fminf(0.f, run + e);
-      run = (k < g) ? nr : run;
-      la[0] = (k == lane) ? run : la[0];
-    }
-    if (nseg > 1) {  // warp-uniform
-#pragma unroll
-      for (int k = 0; k < 32; ++k) {
-        const float e = __shfl_sync(FULL, ellw[1], k);
-        const float nr = fminf(0.f, run + e);
-        run = (32 + k < g) ? nr : run;
-        la[1] = (k == lane) ? run : la[1];
-      }
+#pragma unroll 1
+    for (int k = 0; k < g; ++k) {
+      const float e = __shfl_sync(FULL, k < 32 ? ellw[0] : ellw[1], k & 31);
+      run = fminf(0.f, run + e);
+      if (k < 32) la[0] = (k == lane) ? run : la[0];
+      else la[1] = (k - 32 == lane) ? run : la[1];
     }
     // log alpha_{j-1} of each candidate residual row, and its U-sampler setup
     float lap[2];
@@ -482,7 +473,7 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
       }
 #pragma unroll
       for (int u = 0; u < RU; ++u) {
-        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)(g0 + (int64_t)u * nt), kStreamResid, 0u);
+        const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)(g0 + (int64_t)u * nt), kStreamResid, 0u);
         sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
         sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
         sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
@@ -511,7 +502,7 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
 #pragma unroll
       for (int u = 0; u < RU; ++u) {
         const int64_t gi = g0 + (int64_t)u * nt;
-        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+        const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
         const float g4[4] = {G.x, G.y, G.z, G.w};
         float out[4];
 #pragma unroll
@@ -550,7 +541,7 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
 #pragma unroll
         for (int k = 0; k < 4; ++k) out[k] = a[u][k] - (p[u][k] - q[u][k]) * cs.refl;  // x - delta (1 + 2 S1/S2)
       } else if (draw) {
-        const float4 G = normals4(seed, (uint32_t)b, (uint32_t)gi, bonus ? kStreamBonus : kStreamResid, 0u);
+        const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)gi, bonus ? kStreamBonus : kStreamResid, 0u);
         out[0] = a[u][0] + sgm * G.x; out[1] = a[u][1] + sgm * G.y;
         out[2] = a[u][2] + sgm * G.z; out[3] = a[u][3] + sgm * G.w;
       } else {
@@ -793,9 +784,11 @@ static bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_
 // cudaEventRecordExternal under stream capture, so that they become event-record
 // nodes of the graph (a plain record there only expresses a dependency).
 struct TimingRing {
-  std::vector<cudaEvent_t> ev;  // slots x 4
+  std::vector<cudaEvent_t> ev;  // slots x 3
   int slots = 0;
-  long long next = 0;
+  long long next = 0;   // recorded calls
+  int stride = 1;       // record one call in `stride`
+  long long calls = 0;  // calls seen while enabled
 };
 static thread_local TimingRing g_timing;
 
@@ -804,13 +797,15 @@ static void timing_destroy() {
   g_timing.ev.clear();
   g_timing.slots = 0;
   g_timing.next = 0;
+  g_timing.calls = 0;
 }
 
 static cudaEvent_t* timing_slot() {
   if (g_timing.slots == 0) return nullptr;
+  if (g_timing.calls++ % g_timing.stride != 0) return nullptr;
   const int s = (int)(g_timing.next % g_timing.slots);
   ++g_timing.next;
-  return &g_timing.ev[4 * (size_t)s];
+  return &g_timing.ev[3 * (size_t)s];
 }
 
 static void timing_record(cudaEvent_t e, cudaStream_t s) {
@@ -959,10 +954,7 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
       launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, A.state, part4, y_out, s);
     rc = check_launch();
   }
-  if (tev) {
-    timing_record(tev[2], s);
-    timing_record(tev[3], s);
-  }
+  if (tev) timing_record(tev[2], s);
   return rc;
 }
 
@@ -1103,7 +1095,7 @@ int sdv_timing_enable(int slots) {
   if (slots < 0 || slots > (1 << 20)) return SDV_EINVAL;
   timing_destroy();
   if (slots == 0) return SDV_OK;
-  g_timing.ev.resize(4 * (size_t)slots);
+  g_timing.ev.resize(3 * (size_t)slots);
   for (auto& e : g_timing.ev) {
     if (cudaEventCreate(&e) != cudaSuccess) {
       g_last_cuda_error = (int)cudaGetLastError();
@@ -1115,6 +1107,13 @@ int sdv_timing_enable(int slots) {
   return SDV_OK;
 }
 
+int sdv_timing_stride(int every) {
+  if (every < 1) return SDV_EINVAL;
+  g_timing.stride = every;
+  g_timing.calls = 0;
+  return SDV_OK;
+}
+
 int sdv_timing_read(int n_calls, float* ms3) {
   if (!ms3 || g_timing.slots == 0 || n_calls < 1 || n_calls > g_timing.slots ||
       n_calls > g_timing.next)
@@ -1122,12 +1121,12 @@ int sdv_timing_read(int n_calls, float* ms3) {
   double acc[3] = {0, 0, 0};
   for (int i = 0; i < n_calls; ++i) {
     const int s = (int)((g_timing.next - 1 - i) % g_timing.slots);
-    cudaEvent_t* e = &g_timing.ev[4 * (size_t)s];
-    if (cudaEventSynchronize(e[3]) != cudaSuccess) {
+    cudaEvent_t* e = &g_timing.ev[3 * (size_t)s];
+    if (cudaEventSynchronize(e[2]) != cudaSuccess) {
       g_last_cuda_error = (int)cudaGetLastError();
       return SDV_ECUDA;
     }
-    for (int k = 0; k < 3; ++k) {
+    for (int k = 0; k < 2; ++k) {
       float ms = 0.f;
       if (cudaEventElapsedTime(&ms, e[k], e[k + 1]) != cudaSuccess) {
         g_last_cuda_error = (int)cudaGetLastError();

@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--sampler-L", default="4,8,16",
                    help="draft windows of the end-to-end sampler workload")
     p.add_argument("--mode", default="block", choices=["block", "sample"])
+    p.add_argument("--batch", type=int, default=0,
+                   help="chains per call (0: the workload's B); smaller batches serve ncu captures")
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--skip-cpu", action="store_true")
@@ -303,6 +305,8 @@ def main():
 
     cfg = W.VERIFY_CONFIGS[args.workload]
     Bn, L, d, dt_name = cfg["B"], cfg["L"], cfg["d"], cfg["dtype"]
+    if args.batch > 0:
+        Bn = args.batch
     tdt = torch.bfloat16 if dt_name == "bf16" else torch.float32
     set_bytes = W.main_pass_bytes(Bn, L, d, dt_name)
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size if hasattr(
@@ -317,7 +321,7 @@ def main():
     sets = []
     host0 = None
     for i in range(n_sets):
-        inp = W.make_verify_inputs(args.workload, seed=cfg["seed"] + 100 * i + 7 * rank)
+        inp = W.make_verify_inputs(args.workload, B=Bn, seed=cfg["seed"] + 100 * i + 7 * rank)
         sets.append(dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"),
                          mp=to_dev(inp, "mu_draft"), sigma=torch.from_numpy(inp["sigma"]).to(dev)))
         if i == 0:

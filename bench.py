@@ -457,7 +457,8 @@ def main():
                    "cuda_graph": use_graph},
         "hbm_gbs_step": (set_bytes / (ms_step * 1e-3)) / 1e9,
         "mean_tau_block": taus["block"], "mean_tau_sample": taus["sample"],
-        "phase_us": {"verify_kernel": 1e3 * kv_ms, "long_row_residual": 1e3 * kr_ms},
+        "phase_us": {"verify_kernel": 1e3 * kv_ms,
+                     "long_row_residual": 1e3 * kr_ms if long_rows(d) else None},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                      "kernel": "k_verify (fused: log-ratio pass, acceptance, U-draw%s)"

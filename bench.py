@@ -76,11 +76,12 @@ def kernel_sources_digest():
     return h.hexdigest()
 
 
-def profile_traffic():
-    """dram bytes per launch of the fused verify kernel from the committed ncu summary, if
-    the kernel sources are unchanged since the capture (else None)."""
-    path = os.path.join(ROOT, "profiles", "k_verify_pixel.md")
-    if not os.path.exists(path):
+def profile_traffic(workload, full_size):
+    """dram bytes per launch of the fused verify kernel on this workload from its committed
+    ncu summary, if the kernel sources are unchanged since the capture and the batch is
+    the workload's full one (else None)."""
+    path = os.path.join(ROOT, "profiles", "k_verify_%s.md" % workload)
+    if not full_size or not os.path.exists(path):
         return None
     txt = open(path).read()
     m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
@@ -145,19 +146,29 @@ def long_rows(d):
     return (d + 3) // 4 > FUSED_MAX_GROUPS
 
 
-def launches_per_step(d):
-    """Kernels one sdv_verify call launches: the fused verify kernel, plus the
-    residual dot / write kernels for long rows (the ticket reset is a memset)."""
-    return 3 if long_rows(d) else 1
+# From this many chains on, the library streams the tiles with k_tiles and finishes
+# every chain with one warp of k_finish (the library's kManyChainMin).
+MANY_CHAIN_MIN = 512
+
+
+def many_chains(B):
+    return B >= MANY_CHAIN_MIN
+
+
+def launches_per_step(B, d):
+    """Kernels one sdv_verify call launches: the fused verify kernel (or k_tiles and
+    k_finish for many chains), plus the residual dot / write kernels for long rows
+    (the ticket reset of the fused kernel is a memset)."""
+    return (2 if many_chains(B) else 1) + (2 if long_rows(d) else 0)
 
 
 def fused_kernel_bytes(B, L, d, dtype):
-    """Algorithmic bytes of the fused kernel per call: x, m^q, m^p read once, and, when it
-    also writes the residual, the rejected row's m^q and m^p (upper bound: every chain)
-    re-read plus y written."""
+    """Algorithmic bytes of the first kernel of a call: x, m^q, m^p read once, and, when
+    the fused kernel also writes the residual, the rejected row's m^q and m^p (upper
+    bound: every chain) re-read plus y written."""
     s = W.bytes_per_element(dtype)
     main = 3 * B * L * d * s
-    return main if long_rows(d) else main + 3 * B * d * s
+    return main if (long_rows(d) or many_chains(B)) else main + 3 * B * d * s
 
 
 def dist_setup():
@@ -457,17 +468,20 @@ def main():
                    "cuda_graph": use_graph},
         "hbm_gbs_step": (set_bytes / (ms_step * 1e-3)) / 1e9,
         "mean_tau_block": taus["block"], "mean_tau_sample": taus["sample"],
-        "phase_us": {"verify_kernel": 1e3 * kv_ms,
-                     "long_row_residual": 1e3 * kr_ms if long_rows(d) else None},
+        "phase_us": ({"tiles_kernel": 1e3 * kv_ms, "finish_and_residual": 1e3 * kr_ms}
+                     if many_chains(Bn) else
+                     {"verify_kernel": 1e3 * kv_ms,
+                      "long_row_residual": 1e3 * kr_ms if long_rows(d) else None}),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                     "kernel": "k_verify (fused: log-ratio pass, acceptance, U-draw%s)"
+                     "kernel": "k_tiles (log-ratio pass of the many-chain path)" if many_chains(Bn)
+                               else "k_verify (fused: log-ratio pass, acceptance, U-draw%s)"
                                % ("" if long_rows(d) else ", residual write"),
                      "algorithmic_bytes": kv_bytes,
-                     "traffic": profile_traffic()},
+                     "traffic": profile_traffic(args.workload, Bn == W.VERIFY_CONFIGS[args.workload]["B"])},
         "e2e": {"value": world * Bn * L / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
-        "gpu_launches": launches_per_step(d) * args.steps,
+        "gpu_launches": launches_per_step(Bn, d) * args.steps,
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.skip_cpu:

@@ -284,8 +284,12 @@ size_t sdv_sampler_workspace_bytes(int B, int L, int64_t d);
  * `max_rounds` rounds have run.  One round: gamma_k = min(L, K - k) draft steps, the
  * parallel target call at yhat_k .. yhat_{k+gamma_k}, sdv_verify_ex (residual or bonus
  * step), then k <- min(k + tau, K); a window that reaches K takes no bonus step.
- * Unlike the other entry points this call synchronises: it enqueues the rounds on
- * `stream` and reads the number of active chains back every 8 rounds.
+ * The rounds run as one CUDA graph launched on `stream`: a while node whose body is
+ * one round (draft, target call, verification, update), the round counter and seed
+ * held in the workspace and the loop ended on the device once no chain is active or
+ * max_rounds rounds ran.  Unlike the other entry points this call synchronises (it
+ * waits for the graph to read back the number of rounds), so it cannot itself be
+ * captured into a graph.
  *   y_out [B, d] fp32 out: the chains' states (Y_K when finished)
  *   k_out [B], chain_rounds_out [B], tau_sum_out [B] int32 out or NULL: step reached,
  *     rounds taken part in, sum of tau over those rounds

@@ -14,6 +14,14 @@ constexpr int kK1Vpt = 4;
 // Resident CTAs per SM the fused kernel is built for (its register budget): the
 // chain-finishing code needs more than the streaming loop.
 constexpr int kK1MinBlocks = 3;
+// Many-chain path (B >= kManyChainMin): resident CTAs per SM of the streaming
+// kernel k_tiles (its register budget: 3 x vpt 16-byte buffers per thread), and
+// the finishing kernel k_finish: threads per chain and groups of four elements per
+// thread per residual sweep.
+constexpr int kManyChainMin = 512;
+constexpr int tile_min_blocks(int vpt) { return vpt <= 1 ? 8 : (vpt == 2 ? 6 : 4); }
+constexpr int kFinishThreads = 128;
+constexpr int kFinishResidUnroll = 4;
 // Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;
 // Long-row residual kernels: threads per CTA and elements of the rejected row per CTA.
@@ -57,6 +65,7 @@ struct ScanArgs {
   int B, L;
   const int32_t* L_eff;
   uint64_t seed;
+  const uint64_t* seed_dev;  // nullable: the seed is read from device memory instead
   int mode;
   float inv_omega2;
   int residual_kind;
@@ -81,6 +90,17 @@ struct WsLayout {
 };
 
 WsLayout ws_layout(int B, int L, int64_t d, int dtype);
+
+// sdv_verify_ex with the seed taken from device memory when seed_dev is not null (it
+// is read by the kernels, so a captured call follows the value at replay), and event
+// timing skipped when timed is false.  Same validation and return codes.
+int verify_ex_impl(const void* x_draft, const void* mu_target, const void* mu_draft,
+                   const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                   uint64_t seed, const uint64_t* seed_dev, int mode, const int32_t* L_eff,
+                   const void* mu_target_bonus, const float* sigma_bonus, int residual_kind,
+                   float omega, int32_t* accepted_len, void* y_out, float* log_ratio_out,
+                   float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
+                   void* workspace, size_t workspace_bytes, bool timed, void* stream);
 
 // Records a cudaError_t for sdv_last_cuda_error() (this host thread).
 void set_last_cuda_error(int err);

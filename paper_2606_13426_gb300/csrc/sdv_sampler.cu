@@ -46,116 +46,170 @@ struct Gmm {
   float comp_var;
 };
 
+__host__ __device__ __forceinline__ uint64_t splitmix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Seed of round r: the (r+1)-th SplitMix64 output of a stream started at `seed`.
+__host__ __device__ __forceinline__ uint64_t round_seed(uint64_t seed, int r) {
+  return splitmix64(seed + (uint64_t)(r + 1) * 0x9E3779B97F4A7C15ull);
+}
+
 constexpr int kGmmThreads = 256;              // 8 warps, one state row per warp at a time
 constexpr int kGmmWarps = kGmmThreads / 32;
 constexpr size_t kGmmSmemCap = 96 * 1024;     // stage the means in shared memory up to this size
 
-// m^q and the score for one state row z (generative step k), by one warp.  mu points to
-// the means [C, d] (shared or global memory).  mq / score may be null; z may alias mq:
-// each lane reads a group of four elements before it writes it, and no other lane
-// touches that group.  add_sigma != 0 adds sigma * G (Philox stream noise_stream,
-// sub-counter noise_sub; one Philox block per group of four) to mq.
+// One state row of a target call: state z at generative step k; outputs mq / score
+// (either may be null; z may alias mq: each lane reads a group of four elements
+// before it writes it, and no other lane touches that group).  add_sigma != 0 adds
+// sigma * G to mq (Philox stream noise_stream of chain `chain`, sub-counter k; one
+// Philox block per group of four).
+struct GmmRow {
+  const float* z;
+  float* mq;
+  float* score;
+  int k;
+  uint32_t chain;
+  float add_sigma;
+};
+
+// m^q and the score for nr <= RB rows by one warp: every mean group read from `mu`
+// (shared or global memory) serves all nr rows.  nr is warp-uniform.
 // VEC: d % 4 == 0 and 16-byte aligned rows (float4 accesses); MAXC >= C components.
-template <int MAXC, bool VEC>
-__device__ __forceinline__ void gmm_row_warp(const float* z, int64_t d, int k, const Sched& S,
-                                             const Gmm& G, const float* mu, float* mq, float* score,
-                                             float add_sigma, uint64_t noise_seed,
-                                             uint32_t noise_chain, uint32_t noise_stream,
-                                             uint32_t noise_sub) {
+template <int MAXC, bool VEC, int RB>
+__device__ __forceinline__ void gmm_rows_warp(const GmmRow (&R)[RB], int nr, int64_t d, const Sched& S,
+                                              const Gmm& G, const float* mu, uint64_t noise_seed,
+                                              uint32_t noise_stream) {
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int C = G.C;
-  const float tf = S.tfwd(k);
-  const float ab = S.abar(tf);
-  const float sab = sqrtf(ab);
-  const float v = ab * G.comp_var + 1.0f - ab;
-  const float b = S.beta(tf);
+  float sab[RB], v[RB], be[RB];
+#pragma unroll
+  for (int q = 0; q < RB; ++q) {
+    const float tf = S.tfwd(R[q].k);
+    const float ab = S.abar(tf);
+    sab[q] = sqrtf(ab);
+    v[q] = ab * G.comp_var + 1.0f - ab;
+    be[q] = S.beta(tf);
+  }
   const float cst = 0.5f * (1.0f + S.churn * S.churn);
   const int64_t ng = (d + 3) / 4;
+  // groups in flight per lane: RB rows, times the unrolled sweeps
+  constexpr int kU = RB >= 3 ? 1 : (RB == 2 ? 2 : 4);
   auto load_group = [&](const float* p, int64_t gi, float (&f)[4]) {
     if (VEC) {
       const float4 t = *reinterpret_cast<const float4*>(p + 4 * gi);
       f[0] = t.x; f[1] = t.y; f[2] = t.z; f[3] = t.w;
     } else {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) f[q] = (4 * gi + q < d) ? p[4 * gi + q] : 0.f;
+      for (int e = 0; e < 4; ++e) f[e] = (4 * gi + e < d) ? p[4 * gi + e] : 0.f;
     }
   };
   // pass 1: squared distances to the scaled centres sqrt(abar) mu_c
-  float acc[MAXC];
+  float acc[RB][MAXC];
 #pragma unroll
-  for (int c = 0; c < MAXC; ++c) acc[c] = 0.f;
-#pragma unroll 4
+  for (int q = 0; q < RB; ++q)
+#pragma unroll
+    for (int c = 0; c < MAXC; ++c) acc[q][c] = 0.f;
+#pragma unroll kU
   for (int64_t gi = lane; gi < ng; gi += 32) {
-    float zf[4];
-    load_group(z, gi, zf);
+    float zf[RB][4];
+#pragma unroll
+    for (int q = 0; q < RB; ++q) {
+      if (q < nr) load_group(R[q].z, gi, zf[q]);
+    }
 #pragma unroll
     for (int c = 0; c < MAXC; ++c) {
       if (c < C) {
         float mf[4];
         load_group(mu + (int64_t)c * d, gi, mf);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float df = (4 * gi + q < d) ? zf[q] - sab * mf[q] : 0.f;
-          acc[c] = fmaf(df, df, acc[c]);
+        for (int q = 0; q < RB; ++q) {
+          if (q < nr) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float df = (4 * gi + e < d) ? zf[q][e] - sab[q] * mf[e] : 0.f;
+              acc[q][c] = fmaf(df, df, acc[q][c]);
+            }
+          }
         }
       }
     }
   }
-  // responsibilities r_c = softmax(log w_c - d2_c / (2 v)), identical in every lane
-  float r[MAXC];
-  float mx = -INFINITY;
+  // responsibilities r_c = softmax(log w_c - d2_c / (2 v)), identical in every lane;
+  // acc becomes r, w_sc folds the softmax normaliser and sqrt(abar)
+  float w_sc[RB];
 #pragma unroll
-  for (int c = 0; c < MAXC; ++c) {
-    float a = acc[c];
-    if (c < C) {
+  for (int q = 0; q < RB; ++q) {
+    float mx = -INFINITY;
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(FULL, a, o);
+    for (int c = 0; c < MAXC; ++c) {
+      float a = acc[q][c];
+      if (c < C) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(FULL, a, o);
+      }
+      acc[q][c] = (c < C) ? __ldg(G.log_w + c) - a / (2.0f * v[q]) : -INFINITY;
+      mx = fmaxf(mx, acc[q][c]);
     }
-    r[c] = (c < C) ? __ldg(G.log_w + c) - a / (2.0f * v) : -INFINITY;
-    mx = fmaxf(mx, r[c]);
-  }
-  float den = 0.f;
+    float den = 0.f;
 #pragma unroll
-  for (int c = 0; c < MAXC; ++c) {
-    r[c] = (c < C) ? expf(r[c] - mx) : 0.f;
-    den += r[c];
+    for (int c = 0; c < MAXC; ++c) {
+      acc[q][c] = (c < C) ? expf(acc[q][c] - mx) : 0.f;
+      den += acc[q][c];
+    }
+    w_sc[q] = sab[q] / den;
   }
-  const float w_sc = sab / den;  // folds the softmax normaliser and sqrt(abar)
   // pass 2: score and target mean
-#pragma unroll 4
+#pragma unroll kU
   for (int64_t gi = lane; gi < ng; gi += 32) {
-    float zf[4], wsum[4] = {0.f, 0.f, 0.f, 0.f};
-    load_group(z, gi, zf);
+    float zf[RB][4], wsum[RB][4];
+#pragma unroll
+    for (int q = 0; q < RB; ++q) {
+      if (q < nr) load_group(R[q].z, gi, zf[q]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) wsum[q][e] = 0.f;
+    }
 #pragma unroll
     for (int c = 0; c < MAXC; ++c) {
       if (c < C) {
         float mf[4];
         load_group(mu + (int64_t)c * d, gi, mf);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) wsum[q] = fmaf(r[c], mf[q], wsum[q]);
+        for (int q = 0; q < RB; ++q)
+#pragma unroll
+          for (int e = 0; e < 4; ++e) wsum[q][e] = fmaf(acc[q][c], mf[e], wsum[q][e]);
       }
     }
-    float G4[4] = {0.f, 0.f, 0.f, 0.f};
-    if (add_sigma != 0.f) {
-      const float4 n4 = normals4(noise_seed, noise_chain, (uint32_t)gi, noise_stream, noise_sub);
-      G4[0] = n4.x; G4[1] = n4.y; G4[2] = n4.z; G4[3] = n4.w;
-    }
-    float sc[4], m[4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      sc[q] = (w_sc * wsum[q] - zf[q]) / v;
-      m[q] = zf[q] + S.delta * (0.5f * b * zf[q] + cst * b * sc[q]) + add_sigma * G4[q];
-    }
-    if (VEC) {
-      if (score) *reinterpret_cast<float4*>(score + 4 * gi) = make_float4(sc[0], sc[1], sc[2], sc[3]);
-      if (mq) *reinterpret_cast<float4*>(mq + 4 * gi) = make_float4(m[0], m[1], m[2], m[3]);
-    } else {
+    for (int q = 0; q < RB; ++q) {
+      if (q < nr) {
+        float G4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (R[q].add_sigma != 0.f) {
+          const float4 n4 = normals4(noise_seed, R[q].chain, (uint32_t)gi, noise_stream, (uint32_t)R[q].k);
+          G4[0] = n4.x; G4[1] = n4.y; G4[2] = n4.z; G4[3] = n4.w;
+        }
+        float sc[4], m[4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if (4 * gi + q < d) {
-          if (score) score[4 * gi + q] = sc[q];
-          if (mq) mq[4 * gi + q] = m[q];
+        for (int e = 0; e < 4; ++e) {
+          sc[e] = (w_sc[q] * wsum[q][e] - zf[q][e]) / v[q];
+          m[e] = zf[q][e] + S.delta * (0.5f * be[q] * zf[q][e] + cst * be[q] * sc[e]) + R[q].add_sigma * G4[e];
+        }
+        float* score = R[q].score;
+        float* mq = R[q].mq;
+        if (VEC) {
+          if (score) *reinterpret_cast<float4*>(score + 4 * gi) = make_float4(sc[0], sc[1], sc[2], sc[3]);
+          if (mq) *reinterpret_cast<float4*>(mq + 4 * gi) = make_float4(m[0], m[1], m[2], m[3]);
+        } else {
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            if (4 * gi + e < d) {
+              if (score) score[4 * gi + e] = sc[e];
+              if (mq) mq[4 * gi + e] = m[e];
+            }
+          }
         }
       }
     }
@@ -184,40 +238,71 @@ k_gmm_rows(const float* __restrict__ states, const int32_t* __restrict__ k, cons
   for (int row = blockIdx.x * kGmmWarps + warp; row < n; row += gridDim.x * kGmmWarps) {
     if (mask && mask[row] == 0) continue;
     const int64_t o = (int64_t)row * d;
-    gmm_row_warp<MAXC, VEC>(states + o, d, k[row], S, G, mu, mq ? mq + o : nullptr,
-                            score ? score + o : nullptr, 0.f, 0, 0, 0, 0);
+    const GmmRow R[1] = {{states + o, mq ? mq + o : nullptr, score ? score + o : nullptr, k[row], 0u, 0.f}};
+    gmm_rows_warp<MAXC, VEC, 1>(R, 1, d, S, G, mu, 0, 0);
   }
 }
 
-// Parallel target call of a round, one CTA per chain: state j of chain b is y[b] (j = 0)
-// or x_draft[b, j-1], at step k[b] + j, for j = 0 .. gamma_b.  Means go to mu_target[b, j]
-// (j < gamma_b) or mu_bonus[b] (j = gamma_b, with sigma_bonus[b] = sigma_{k+gamma});
-// scores to sc_all[b, j].
+// Rows of a round's parallel target call per warp.
+template <int MAXC> struct RoundRows { static constexpr int value = MAXC <= 8 ? 3 : 2; };
+
+// Parallel target call of a round.  Row (b, j), j = 0 .. gamma_b, is state y[b]
+// (j = 0) or x_draft[b, j-1] at step k[b] + j; its mean goes to mu_target[b, j]
+// (j < gamma_b) or mu_bonus[b] (j = gamma_b, with sigma_bonus[b] = sigma_{k+gamma}),
+// its score to sc_all[b, j].  The B (L+1) row slots are dealt to warps RB at a time
+// (slots past gamma_b are skipped), grid-stride over persistent CTAs.
 template <int MAXC, bool VEC>
-__global__ void __launch_bounds__(kGmmThreads)
+__global__ void __launch_bounds__(kGmmThreads, 2)
 k_round_target(const float* __restrict__ y, const float* __restrict__ x_draft,
-               const int32_t* __restrict__ kk, const int32_t* __restrict__ gam, int L, int64_t d,
+               const int32_t* __restrict__ kk, const int32_t* __restrict__ gam, int B, int L, int64_t d,
                Sched S, Gmm G, bool use_smem, float* mu_target, float* mu_bonus, float* sigma_bonus,
                float* sc_all) {
-  const int b = blockIdx.x;
-  const int g = gam[b];
-  if (g == 0) return;  // CTA-uniform: before any barrier
+  constexpr int RB = RoundRows<MAXC>::value;
   const float* mu = stage_means(G, d, use_smem);
-  const int warp = threadIdx.x >> 5;
-  for (int j = warp; j <= g; j += kGmmWarps) {
-    const float* z = (j == 0) ? y + (int64_t)b * d : x_draft + ((int64_t)b * L + j - 1) * d;
-    float* mq = (j < g) ? mu_target + ((int64_t)b * L + j) * d : mu_bonus + (int64_t)b * d;
-    gmm_row_warp<MAXC, VEC>(z, d, kk[b] + j, S, G, mu, mq, sc_all + ((int64_t)b * (L + 1) + j) * d,
-                            0.f, 0, 0, 0, 0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t slots = (int64_t)B * (L + 1);
+  for (int64_t r0 = ((int64_t)blockIdx.x * kGmmWarps + warp) * RB; r0 < slots;
+       r0 += (int64_t)gridDim.x * kGmmWarps * RB) {
+    GmmRow R[RB];
+    int nr = 0;
+#pragma unroll
+    for (int q = 0; q < RB; ++q) {
+      R[q] = GmmRow{nullptr, nullptr, nullptr, 0, 0u, 0.f};
+      const int64_t slot = r0 + q;
+      if (slot >= slots) continue;
+      const int b = (int)(slot / (L + 1));
+      const int j = (int)(slot - (int64_t)b * (L + 1));
+      const int g = gam[b];
+      if (j > g || g == 0) continue;
+      const int kb = kk[b];
+      GmmRow row;
+      row.z = (j == 0) ? y + (int64_t)b * d : x_draft + ((int64_t)b * L + j - 1) * d;
+      row.mq = (j < g) ? mu_target + ((int64_t)b * L + j) * d : mu_bonus + (int64_t)b * d;
+      row.score = sc_all + ((int64_t)b * (L + 1) + j) * d;
+      row.k = kb + j;
+      row.chain = 0u;
+      row.add_sigma = 0.f;
+      if (j == g && lane == 0) sigma_bonus[b] = S.sigma(kb + g);
+      // compact the live rows to the front (q is a compile-time index after unrolling)
+#pragma unroll
+      for (int t = 0; t < RB; ++t)
+        if (t == nr) R[t] = row;
+      ++nr;
+    }
+    if (nr > 0) gmm_rows_warp<MAXC, VEC, RB>(R, nr, d, S, G, mu, 0, 0);
   }
-  if (threadIdx.x == 0) sigma_bonus[b] = S.sigma(kk[b] + g);
 }
 
 // Free / Frozen drafter: gamma_b elementwise steps from y[b] with the cached score.
+// One thread per group of four elements; VEC: d % 4 == 0 and 16-byte aligned rows
+// (float4 loads and stores).  The Philox draws do not depend on the state, so the
+// unrolled step loop overlaps the next step's draws with this step's stores.
+template <bool VEC>
 __global__ void __launch_bounds__(256)
 k_draft(const float* __restrict__ y, const float* __restrict__ s_cache, const int32_t* __restrict__ kk,
-        const int32_t* __restrict__ gam, int B, int L, int64_t d, Sched S, uint64_t seed,
-        float* x_draft, float* mu_draft, float* sigma) {
+        const int32_t* __restrict__ gam, int B, int L, int64_t d, Sched S, uint64_t seed_v,
+        const uint64_t* __restrict__ seed_dev, float* __restrict__ x_draft, float* __restrict__ mu_draft,
+        float* __restrict__ sigma) {
   const int64_t ng = (d + 3) / 4;
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * ng) return;
@@ -225,15 +310,24 @@ k_draft(const float* __restrict__ y, const float* __restrict__ s_cache, const in
   const int64_t gi = t - (int64_t)b * ng;
   const int g = gam[b];
   if (g == 0) return;
+  const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int k = kk[b];
   const float cst = 0.5f * (1.0f + S.churn * S.churn);
+  const int64_t i0 = 4 * gi;
   float cur[4], sc[4];
+  if (VEC) {
+    const float4 a = *reinterpret_cast<const float4*>(y + (int64_t)b * d + i0);
+    const float4 c = *reinterpret_cast<const float4*>(s_cache + (int64_t)b * d + i0);
+    cur[0] = a.x; cur[1] = a.y; cur[2] = a.z; cur[3] = a.w;
+    sc[0] = c.x; sc[1] = c.y; sc[2] = c.z; sc[3] = c.w;
+  } else {
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const int64_t i = 4 * gi + q;
-    cur[q] = (i < d) ? y[(int64_t)b * d + i] : 0.f;
-    sc[q] = (i < d) ? s_cache[(int64_t)b * d + i] : 0.f;
+    for (int q = 0; q < 4; ++q) {
+      cur[q] = (i0 + q < d) ? y[(int64_t)b * d + i0 + q] : 0.f;
+      sc[q] = (i0 + q < d) ? s_cache[(int64_t)b * d + i0 + q] : 0.f;
+    }
   }
+#pragma unroll 4
   for (int step = 1; step <= g; ++step) {
     const int kc = k + step - 1;
     const float be = S.beta(S.tfwd(kc));
@@ -241,16 +335,23 @@ k_draft(const float* __restrict__ y, const float* __restrict__ s_cache, const in
     const float4 n4 = normals4(seed, (uint32_t)b, (uint32_t)gi, kStreamDraft, (uint32_t)(step - 1));
     const float nz[4] = {n4.x, n4.y, n4.z, n4.w};
     const int64_t row = ((int64_t)b * L + step - 1) * d;
+    float m[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const int64_t i = 4 * gi + q;
-      const float m = cur[q] + S.delta * (0.5f * be * cur[q] + cst * be * sc[q]);
-      const float nx = m + sg * nz[q];
-      if (i < d) {
-        mu_draft[row + i] = m;
-        x_draft[row + i] = nx;
+      m[q] = cur[q] + S.delta * (0.5f * be * cur[q] + cst * be * sc[q]);
+      cur[q] = m[q] + sg * nz[q];
+    }
+    if (VEC) {
+      *reinterpret_cast<float4*>(mu_draft + row + i0) = make_float4(m[0], m[1], m[2], m[3]);
+      *reinterpret_cast<float4*>(x_draft + row + i0) = make_float4(cur[0], cur[1], cur[2], cur[3]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        if (i0 + q < d) {
+          mu_draft[row + i0 + q] = m[q];
+          x_draft[row + i0 + q] = cur[q];
+        }
       }
-      cur[q] = nx;
     }
     if (gi == 0) sigma[(int64_t)b * L + step - 1] = sg;
   }
@@ -287,9 +388,28 @@ k_round_update(const int32_t* __restrict__ acc, const float* __restrict__ y_out,
   }
 }
 
+// Device-resident state of the round loop: the seed of the current round, the rounds
+// run, and the chains k_round_update found still active in the current round.
+struct SamplerCtl {
+  uint64_t seed_r;
+  int32_t r;
+  uint32_t active;
+};
+
+// End of a round (one thread): advance the round counter and seed, and keep the loop
+// of the round graph going while a chain is active and fewer than max_rounds ran.
+__global__ void k_round_close(SamplerCtl* ctl, uint64_t seed, int max_rounds, cudaGraphConditionalHandle h) {
+  const int r = ctl->r + 1;
+  ctl->r = r;
+  ctl->seed_r = round_seed(seed, r);
+  const bool more = ctl->active != 0u && r < max_rounds;
+  ctl->active = 0u;
+  cudaGraphSetConditional(h, more ? 1u : 0u);
+}
+
 __global__ void __launch_bounds__(256)
 k_sampler_init(int B, int L, int64_t d, int K, uint64_t seed, float* y, int32_t* kk, int32_t* gam,
-               int32_t* rounds, int32_t* tau_sum) {
+               int32_t* rounds, int32_t* tau_sum, SamplerCtl* ctl) {
   const int64_t ng = (d + 3) / 4;
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= (int64_t)B * ng) return;
@@ -300,6 +420,11 @@ k_sampler_init(int B, int L, int64_t d, int K, uint64_t seed, float* y, int32_t*
 #pragma unroll
   for (int q = 0; q < 4; ++q)
     if (4 * gi + q < d) y[(int64_t)b * d + 4 * gi + q] = nz[q];
+  if (t == 0 && ctl != nullptr) {
+    ctl->seed_r = round_seed(seed, 0);
+    ctl->r = 0;
+    ctl->active = 0u;
+  }
   if (gi == 0 && kk != nullptr) {
     kk[b] = 0;
     gam[b] = min(L, K);
@@ -317,8 +442,8 @@ k_em_step(float* y, int B, int64_t d, int k, Sched S, Gmm G, bool use_smem, uint
   const int warp = threadIdx.x >> 5;
   for (int b = blockIdx.x * kGmmWarps + warp; b < B; b += gridDim.x * kGmmWarps) {
     float* row = y + (int64_t)b * d;
-    gmm_row_warp<MAXC, VEC>(row, d, k, S, G, mu, row, nullptr, S.sigma(k), seed, (uint32_t)b, kStreamEM,
-                            (uint32_t)k);
+    const GmmRow R[1] = {{row, row, nullptr, k, (uint32_t)b, S.sigma(k)}};
+    gmm_rows_warp<MAXC, VEC, 1>(R, 1, d, S, G, mu, seed, kStreamEM);
   }
 }
 
@@ -355,6 +480,25 @@ static GmmLaunch gmm_launch(int C, int64_t d, const void* means, bool rows_align
 
 static unsigned rows_grid(int n) { return (unsigned)std::max(1, (n + kGmmWarps - 1) / kGmmWarps); }
 
+static int sm_count() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  if (cache[dev] == 0) {
+    int n = 0;
+    cache[dev] = (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0) ? n : 152;
+  }
+  return cache[dev];
+}
+
+// Grid of k_round_target: one warp per RB row slots, at most four CTAs per SM (each
+// CTA stages the means once and strides over its share of the slots).
+static unsigned round_target_grid(const GmmLaunch& gl, int B, int L) {
+  const int64_t rb = gl.maxc <= 8 ? RoundRows<8>::value : RoundRows<16>::value;
+  const int64_t need = ((int64_t)B * (L + 1) + kGmmWarps * rb - 1) / (kGmmWarps * rb);
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, 4 * (int64_t)sm_count()));
+}
+
 #define SDV_GMM_DISPATCH(GL, KERNEL, GRID, STREAM, ...)                                          \
   do {                                                                                          \
     if ((GL).maxc == 8) {                                                                       \
@@ -375,17 +519,6 @@ static int launch_check() {
   return SDV_OK;
 }
 
-static uint64_t splitmix64(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
-// Seed of round r: the (r+1)-th SplitMix64 output of a stream started at `seed`.
-static uint64_t round_seed(uint64_t seed, int r) {
-  return splitmix64(seed + (uint64_t)(r + 1) * 0x9E3779B97F4A7C15ull);
-}
-
 static bool valid_sched(int K, float churn, float bmin, float bmax, float tfl) {
   return K >= 1 && std::isfinite(churn) && churn > 0.f && std::isfinite(bmin) && std::isfinite(bmax) &&
          bmin > 0.f && bmax >= bmin && tfl > 0.f && tfl <= 1.f;
@@ -399,7 +532,7 @@ static Sched make_sched(int K, float churn, float bmin, float bmax, float tfl) {
 }
 
 struct SamplerLayout {
-  size_t y, s, k, g, x, mp, mq, mqb, sg, sgb, sc, acc, yo, rounds, tausum, active, vws, total;
+  size_t y, s, k, g, x, mp, mq, mqb, sg, sgb, sc, acc, yo, rounds, tausum, ctl, vws, total;
 };
 
 static SamplerLayout sampler_layout(int B, int L, int64_t d) {
@@ -423,7 +556,7 @@ static SamplerLayout sampler_layout(int B, int L, int64_t d) {
   w.yo = o; o = up(o + Bd);
   w.rounds = o; o = up(o + (size_t)B * 4);
   w.tausum = o; o = up(o + (size_t)B * 4);
-  w.active = o; o = up(o + 4);
+  w.ctl = o; o = up(o + sizeof(SamplerCtl));
   w.vws = o; o = up(o + sdv_workspace_bytes(B, L, d, SDV_F32));
   w.total = o;
   return w;
@@ -463,8 +596,12 @@ int sdv_free_draft(const float* y, const float* score, const int32_t* k, const i
   if (!valid_sched(K, churn, beta_min, beta_max, t_floor)) return SDV_EINVAL;
   const Sched S = make_sched(K, churn, beta_min, beta_max, t_floor);
   const int64_t n = (int64_t)B * ((d + 3) / 4);
-  k_draft<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(y, score, k, L_eff, B, L, d, S, seed,
-                                                                         x_draft, mu_draft, sigma);
+  const bool vec = (d % 4 == 0) && ((reinterpret_cast<uintptr_t>(y) | reinterpret_cast<uintptr_t>(score) |
+                                      reinterpret_cast<uintptr_t>(x_draft) |
+                                      reinterpret_cast<uintptr_t>(mu_draft)) % 16 == 0);
+  const unsigned grid = (unsigned)((n + 255) / 256);
+  if (vec) k_draft<true><<<grid, 256, 0, (cudaStream_t)stream>>>(y, score, k, L_eff, B, L, d, S, seed, nullptr, x_draft, mu_draft, sigma);
+  else k_draft<false><<<grid, 256, 0, (cudaStream_t)stream>>>(y, score, k, L_eff, B, L, d, S, seed, nullptr, x_draft, mu_draft, sigma);
   return launch_check();
 }
 
@@ -505,7 +642,7 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
   float* yo = (float*)(ws + w.yo);
   int32_t* rounds = (int32_t*)(ws + w.rounds);
   int32_t* tsum = (int32_t*)(ws + w.tausum);
-  unsigned int* active = (unsigned int*)(ws + w.active);
+  SamplerCtl* ctl = (SamplerCtl*)(ws + w.ctl);
   void* vws = ws + w.vws;
   const size_t vws_bytes = w.total - w.vws;
   const Sched S = make_sched(K, churn, beta_min, beta_max, t_floor);
@@ -516,42 +653,80 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
   const GmmLaunch gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(workspace) % 16 == 0);
 
   int rc;
-  k_sampler_init<<<eg, 256, 0, s>>>(B, L, d, K, seed, y, kk, gam, rounds, tsum);
+  k_sampler_init<<<eg, 256, 0, s>>>(B, L, d, K, seed, y, kk, gam, rounds, tsum, ctl);
   if ((rc = launch_check()) != SDV_OK) return rc;
   // the only explicit target call: the score at Y_0 (step 0)
   SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), s, y, kk, nullptr, B, d, S, G, gl.smem, nullptr, sc);
   if ((rc = launch_check()) != SDV_OK) return rc;
 
-  int r = 0;
-  const int check_every = 8;
-  for (; r < max_rounds; ++r) {
-    const uint64_t seed_r = round_seed(seed, r);
-    if (drafter == SDV_DRAFTER_FROZEN) {  // a fresh score at the round's start state
-      SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), s, y, kk, gam, B, d, S, G, gl.smem, nullptr, sc);
-      if ((rc = launch_check()) != SDV_OK) return rc;
+  // The round loop is one CUDA graph: a while node whose body is one round, captured
+  // once; the round's seed lives in device memory (SamplerCtl) and k_round_close ends
+  // the loop.  One graph launch runs every round with no host round trip.
+  if (max_rounds > 0) {
+    cudaGraph_t graph = nullptr, body = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    cudaStream_t cs = nullptr;
+    cudaGraphConditionalHandle handle = 0;
+    cudaGraphNode_t loop = nullptr;
+    bool ok = cudaGraphCreate(&graph, 0) == cudaSuccess &&
+              cudaGraphConditionalHandleCreate(&handle, graph, 1u, cudaGraphCondAssignDefault) == cudaSuccess;
+    if (ok) {
+      cudaGraphNodeParams cp{};
+      cp.type = cudaGraphNodeTypeConditional;
+      cp.conditional.handle = handle;
+      cp.conditional.type = cudaGraphCondTypeWhile;
+      cp.conditional.size = 1;
+      ok = cudaGraphAddNode(&loop, graph, nullptr, nullptr, 0, &cp) == cudaSuccess;
+      if (ok) body = cp.conditional.phGraph_out[0];
     }
-    k_draft<<<eg, 256, 0, s>>>(y, sc, kk, gam, B, L, d, S, seed_r, xd, mpd, sg);
-    if ((rc = launch_check()) != SDV_OK) return rc;
-    SDV_GMM_DISPATCH(gl, k_round_target, B, s, y, xd, kk, gam, L, d, S, G, gl.smem, mqd, mqb, sgb, scall);
-    if ((rc = launch_check()) != SDV_OK) return rc;
-    rc = sdv_verify_ex(xd, mqd, mpd, sg, L, B, L, d, SDV_F32, seed_r, mode, gam, mqb, sgb,
-                       SDV_RESIDUAL_DECOMPOSITION, 1.0f, acc, yo, nullptr, nullptr, nullptr, nullptr,
-                       vws, vws_bytes, stream);
-    if (rc != SDV_OK) return rc;
-    if (cudaMemsetAsync(active, 0, sizeof(unsigned int), s) != cudaSuccess) return launch_check(), SDV_ECUDA;
-    k_round_update<<<B, 256, 0, s>>>(acc, yo, xd, scall, L, d, K, y, sc, kk, gam, rounds, tsum, active);
-    if ((rc = launch_check()) != SDV_OK) return rc;
-    if ((r + 1) % check_every == 0 || r + 1 == max_rounds) {
-      unsigned int h_active = 1;
-      if (cudaMemcpyAsync(&h_active, active, sizeof(h_active), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-          cudaStreamSynchronize(s) != cudaSuccess)
-        return launch_check(), SDV_ECUDA;
-      if (h_active == 0) {
-        ++r;
-        break;
+    ok = ok && cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal) ==
+             cudaSuccess;
+    if (ok) {
+      rc = SDV_OK;
+      if (drafter == SDV_DRAFTER_FROZEN) {  // a fresh score at the round's start state
+        SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), cs, y, kk, gam, B, d, S, G, gl.smem, nullptr, sc);
+        rc = launch_check();
       }
+      if (rc == SDV_OK) {
+        if (gl.vec) k_draft<true><<<eg, 256, 0, cs>>>(y, sc, kk, gam, B, L, d, S, 0, &ctl->seed_r, xd, mpd, sg);
+        else k_draft<false><<<eg, 256, 0, cs>>>(y, sc, kk, gam, B, L, d, S, 0, &ctl->seed_r, xd, mpd, sg);
+        rc = launch_check();
+      }
+      if (rc == SDV_OK) {
+        SDV_GMM_DISPATCH(gl, k_round_target, round_target_grid(gl, B, L), cs, y, xd, kk, gam, B, L, d, S, G,
+                         gl.smem, mqd, mqb, sgb, scall);
+        rc = launch_check();
+      }
+      if (rc == SDV_OK)
+        rc = verify_ex_impl(xd, mqd, mpd, sg, L, B, L, d, SDV_F32, 0, &ctl->seed_r, mode, gam, mqb, sgb,
+                            SDV_RESIDUAL_DECOMPOSITION, 1.0f, acc, yo, nullptr, nullptr, nullptr, nullptr,
+                            vws, vws_bytes, false, cs);
+      if (rc == SDV_OK) {
+        k_round_update<<<B, 256, 0, cs>>>(acc, yo, xd, scall, L, d, K, y, sc, kk, gam, rounds, tsum, &ctl->active);
+        rc = launch_check();
+      }
+      if (rc == SDV_OK) {
+        k_round_close<<<1, 1, 0, cs>>>(ctl, seed, max_rounds, handle);
+        rc = launch_check();
+      }
+      cudaGraph_t captured = nullptr;
+      const bool ended = cudaStreamEndCapture(cs, &captured) == cudaSuccess;
+      ok = rc == SDV_OK && ended && cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess &&
+           cudaGraphLaunch(exec, s) == cudaSuccess;
+    }
+    if (exec) cudaGraphExecDestroy(exec);
+    if (graph) cudaGraphDestroy(graph);
+    if (cs) cudaStreamDestroy(cs);
+    if (!ok) {
+      if (rc != SDV_OK) return rc;
+      return launch_check(), SDV_ECUDA;
     }
   }
+  int r = 0;
+  if (cudaMemcpyAsync(&r, &ctl->r, sizeof(r), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
   *rounds_out = r;
   if (cudaMemcpyAsync(y_out, y, (size_t)B * d * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
     return launch_check(), SDV_ECUDA;
@@ -577,7 +752,7 @@ int sdv_em_sample(int B, int64_t d, const float* means, const float* log_weights
   const int64_t ng = (int64_t)B * ((d + 3) / 4);
   // the initial state only needs y; the bookkeeping arrays of the init kernel are not used
   k_sampler_init<<<(unsigned)((ng + 255) / 256), 256, 0, s>>>(B, 1, d, K, seed, y_out, nullptr, nullptr,
-                                                              nullptr, nullptr);
+                                                              nullptr, nullptr, nullptr);
   int rc = launch_check();
   if (rc != SDV_OK) return rc;
   const GmmLaunch gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(y_out) % 16 == 0);

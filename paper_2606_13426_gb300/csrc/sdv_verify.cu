@@ -15,7 +15,8 @@
 // Chains finish at staggered times, so the latency-bound per-chain work overlaps
 // the streaming of other chains.  Rows longer than kFusedMaxGroups groups of four
 // elements are written by two extra kernels (k_resid_dot, k_resid_write) spread
-// over many CTAs.
+// over many CTAs.  With many chains (B >= kManyChainMin) the same tiles are
+// streamed by k_tiles and every chain is finished by a small CTA of k_finish.
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
@@ -178,6 +179,9 @@ __device__ __forceinline__ float2 tile_sums(const T* __restrict__ x, const T* __
   return make_float2(s1, s2);
 }
 
+// The verification seed: by value, or from device memory (sampler rounds).
+__device__ __forceinline__ uint64_t seed_of(const ScanArgs& A) { return A.seed_dev ? *A.seed_dev : A.seed; }
+
 // ---------------------------------------------------------------- chain scan (one warp)
 __device__ __forceinline__ ChainState inactive_state() {
   ChainState cs;
@@ -283,7 +287,7 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
     const int j = lane + 32 * q;
     leta[q] = 0.f;
     if (q < nseg && j < g)
-      leta[q] = log_uniform(philox_block(A.seed, (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
+      leta[q] = log_uniform(philox_block(seed_of(A), (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
   }
   const float ellw[2] = {ell[0] * A.inv_omega2, ell[1] * A.inv_omega2};
 
@@ -417,19 +421,10 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
   return out;
 }
 
-// Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch), then
-// the outputs that depend on it: status bits and (U, log alpha_res, |Delta_tau|, sigma_tau).
-template <int NT>
-__device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, ChainState& cs,
-                                                  const UParams* P, USampleScratch* us) {
-  if (cs.kind == kKindResid && A.draw_u) {
-    const uint32_t wbits = philox_block(A.seed, (uint32_t)b, 0u, kStreamUSample, 0u).x;
-    uint32_t st = cs.status;
-    const UParams Q = P ? *P : usample_setup(cs.dnorm, fminf(cs.la_res, 0.f));
-    cs.U = usample_block<NT>(Q, wbits, &st, us);
-    cs.status = st;
-  }
-  if (threadIdx.x == 0 && cs.kind != kKindInactive) {
+// Per-chain outputs that depend on U: status bits and (U, log alpha_res, |Delta_tau|,
+// sigma_tau); written by one thread (leader).
+__device__ __forceinline__ void report_chain(const ScanArgs& A, int b, const ChainState& cs, bool leader) {
+  if (leader && cs.kind != kKindInactive) {
     if (A.status_out) A.status_out[b] = cs.status;
     if (A.aux_out) {
       float* a = A.aux_out + 4 * (int64_t)b;
@@ -441,58 +436,67 @@ __device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, Chai
   }
 }
 
-// ---------------------------------------------------------------- residual row by one CTA
-// Writes y[b, :] for chain state cs with the whole CTA (blockDim.x threads, a
-// multiple of 32).  Decomposition: pass A reduces delta^T G, pass B writes
-// m^q + sigma (G + e (U - e^T G)), drawing G again (same Philox counters) rather
-// than holding the row on chip.  Each thread handles kResidUnroll groups of four
-// elements per sweep, loads and Philox blocks of all of them issued together.
-constexpr int kResidUnroll = 1;
+// Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch), then
+// the chain's reported outputs.
+template <int NT>
+__device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, ChainState& cs,
+                                                  const UParams* P, USampleScratch* us) {
+  if (cs.kind == kKindResid && A.draw_u) {
+    const uint32_t wbits = philox_block(seed_of(A), (uint32_t)b, 0u, kStreamUSample, 0u).x;
+    uint32_t st = cs.status;
+    const UParams Q = P ? *P : usample_setup(cs.dnorm, fminf(cs.la_res, 0.f));
+    cs.U = usample_block<NT>(Q, wbits, &st, us);
+    cs.status = st;
+  }
+  report_chain(A, b, cs, threadIdx.x == 0);
+}
 
-template <typename T, bool VEC4>
-__device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
+// ---------------------------------------------------------------- residual row
+// The thread group that writes one residual row: a whole CTA (the fused kernel's
+// finishing CTA, or k_finish's).  all_sum returns the group's sum in every thread,
+// reduced lane-wise within warps, then over warps in warp order.
+struct CtaGroup {
+  float2* red;   // [blockDim.x / 32]
+  float* bcast;
+  __device__ __forceinline__ int rank() const { return threadIdx.x; }
+  __device__ __forceinline__ int size() const { return blockDim.x; }
+  __device__ __forceinline__ float all_sum(float v) const {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5].x = v;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      float w = (threadIdx.x < blockDim.x / 32) ? red[threadIdx.x].x : 0.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
+      if (threadIdx.x == 0) *bcast = w;
+    }
+    __syncthreads();
+    return *bcast;
+  }
+};
+
+// Writes y[b, :] for chain state cs with the threads of group grp (every thread of
+// the group calls it with the same cs).  Decomposition: pass A reduces delta^T G,
+// pass B writes m^q + sigma (G + e (U - e^T G)).  With gcache (room for the row's
+// groups, used only by the thread that owns a group) pass A keeps G there for pass
+// B (GCACHE); without it pass B draws G again (same Philox counters).  Each thread handles RU
+// groups of four elements per sweep, the loads of all of them issued before any use.
+template <typename T, bool VEC4, int RU, bool GCACHE, typename Group>
+__device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
                              const T* __restrict__ mp, const T* __restrict__ mq_bonus,
                              const float* __restrict__ sigma_bonus, int L, int64_t d,
                              uint64_t seed, int b, const ChainState& cs, T* __restrict__ y,
-                             float2* red, float* bcast) {
+                             const Group& grp, float4* gcache) {
   if (cs.kind == kKindInactive) return;
-  constexpr int RU = kResidUnroll;
-  const int nt = blockDim.x;
+  const int nt = grp.size();
   const int64_t ng = (d + 3) / 4;
   const int64_t rbase = ((int64_t)b * L + cs.row) * d;
   const int64_t ybase = (int64_t)b * d;
   // groups past the row end load zeros (load4 guards each element) and store nothing
   if (cs.kind == kKindResid) {
     float sp = 0.f;
-    for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
-      float fq[RU][4], fp[RU][4];
-#pragma unroll
-      for (int u = 0; u < RU; ++u) {
-        load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
-        load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < RU; ++u) {
-        const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)(g0 + (int64_t)u * nt), kStreamResid, 0u);
-        sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
-        sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
-        sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
-        sp = fmaf(fp[u][3] - fq[u][3], G.w, sp);
-      }
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sp += __shfl_xor_sync(0xffffffffu, sp, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5].x = sp;
-    __syncthreads();
-    if (threadIdx.x < 32) {
-      float v = (threadIdx.x < nt / 32) ? red[threadIdx.x].x : 0.f;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-      if (threadIdx.x == 0) *bcast = cs.U - v * cs.inv_norm;  // U - e^T G
-    }
-    __syncthreads();
-    const float coef = *bcast;
-    for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
+    for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
       float fq[RU][4], fp[RU][4];
 #pragma unroll
       for (int u = 0; u < RU; ++u) {
@@ -503,6 +507,26 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
       for (int u = 0; u < RU; ++u) {
         const int64_t gi = g0 + (int64_t)u * nt;
         const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+        if (GCACHE && gi < ng) gcache[gi] = G;
+        sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
+        sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
+        sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
+        sp = fmaf(fp[u][3] - fq[u][3], G.w, sp);
+      }
+    }
+    const float coef = cs.U - grp.all_sum(sp) * cs.inv_norm;  // U - e^T G
+    for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
+      float fq[RU][4], fp[RU][4];
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
+        load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < RU; ++u) {
+        const int64_t gi = g0 + (int64_t)u * nt;
+        const float4 G = GCACHE ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
+                                : normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
         const float g4[4] = {G.x, G.y, G.z, G.w};
         float out[4];
 #pragma unroll
@@ -516,7 +540,7 @@ __device__ void residual_cta(const T* __restrict__ x, const T* __restrict__ mq,
   const bool bonus = cs.kind == kKindBonus;
   const bool draw = bonus || cs.kind == kKindZeroDelta;
   const float sgm = bonus ? sigma_bonus[b] : cs.sigma;
-  for (int64_t g0 = threadIdx.x; g0 < ng; g0 += (int64_t)nt * RU) {
+  for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
     float a[RU][4], q[RU][4], p[RU][4];
 #pragma unroll
     for (int u = 0; u < RU; ++u) {
@@ -626,9 +650,68 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   if (RESID == 0) {
     if (threadIdx.x == 0) A.state[b] = cs;
   } else {
-    residual_cta<T, VEC4>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, A.S.seed, b,
-                          cs, (T*)A.y, red, &bcast);
+    residual_row<T, VEC4, 1, false>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
+                                    b, cs, (T*)A.y, CtaGroup{red, &bcast}, nullptr);
   }
+}
+
+// ---------------------------------------------------------------- many-chain path
+// With many chains the fused kernel's finishing CTAs (each holding a CTA slot for
+// the whole latency-bound scan / U-draw / residual) take more SM time than the
+// stream itself.  The many-chain path streams the same tiles without tickets
+// (k_tiles: identical partials) at full occupancy, then finishes every chain with
+// a small CTA (k_finish: one warp's scan and U-draw, then the residual row), all
+// chains at once.
+template <typename T, bool VEC, int VPT>
+__global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(VerifyArgs A) {
+  __shared__ float2 red[kK1Threads / 32];
+  const int L = A.S.L;
+  const int C = A.S.C;
+  const int64_t tile = blockIdx.x;
+  const int64_t r = tile / C;
+  const int c = (int)(tile - r * C);
+  const int b = (int)(r / L), j = (int)(r - (int64_t)b * L);
+  const int g = A.S.L_eff ? max(0, min(A.S.L_eff[b], L)) : L;
+  if (j >= g) return;  // CTA-uniform
+  const int64_t e0 = (int64_t)c * A.chunk;
+  const int64_t e1 = min(e0 + A.chunk, A.d);
+  const float2 s = tile_sums<T, VEC, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
+  const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
+  if (threadIdx.x == 0) A.part[tile] = t;
+}
+
+// One CTA per chain: warp 0 scans the chain and draws U (warp U-sampler); then, with
+// RESID = 1, all kFinishThreads threads write y (launched with 32 threads and
+// leaving the chain state for k_resid_* when RESID = 0).
+template <typename T, bool VEC4, int RESID>
+__global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
+  __shared__ ChainState cs_s;
+  __shared__ float2 red[kFinishThreads / 32];
+  __shared__ float bcast;
+  __shared__ float4 g_s[RESID ? kFusedMaxGroups : 1];  // the residual's G, drawn once
+  const int b = blockIdx.x;
+  if (threadIdx.x < 32) {
+    const ScanOut so = scan_warp(A.S, b);
+    ChainState cs = so.cs;
+    if (cs.kind == kKindResid && A.S.draw_u) {
+      const uint32_t wbits = philox_block(seed_of(A.S), (uint32_t)b, 0u, kStreamUSample, 0u).x;
+      uint32_t st = cs.status;
+      const UParams Q = so.have_P ? so.P : usample_setup(cs.dnorm, fminf(cs.la_res, 0.f));
+      cs.U = usample_warp(Q, wbits, &st);
+      cs.status = st;
+    }
+    report_chain(A.S, b, cs, threadIdx.x == 0);
+    if (threadIdx.x == 0) {
+      if (RESID == 0) A.state[b] = cs;
+      else cs_s = cs;
+    }
+  }
+  if (RESID == 0) return;
+  __syncthreads();
+  const ChainState cs = cs_s;
+  residual_row<T, VEC4, kFinishResidUnroll, true>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
+                                            (const T*)A.mq_bonus, A.sigma_bonus, A.S.L, A.d, seed_of(A.S),
+                                            b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
 }
 
 // ---------------------------------------------------------------- acceptance scan only
@@ -642,8 +725,10 @@ __global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
 template <typename T, bool VEC4>
 __global__ void __launch_bounds__(kK4Threads)
 k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d, int C4,
-            uint64_t seed, const ChainState* __restrict__ state, float* __restrict__ part4) {
+            uint64_t seed_v, const uint64_t* __restrict__ seed_dev, const ChainState* __restrict__ state,
+            float* __restrict__ part4) {
   __shared__ float2 red[kK4Threads / 32];
+  const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
   const ChainState cs = state[b];
   if (cs.kind != kKindResid) return;
@@ -669,8 +754,9 @@ template <typename T, bool VEC4>
 __global__ void __launch_bounds__(kK4Threads)
 k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __restrict__ mp,
               const T* __restrict__ mq_bonus, const float* __restrict__ sigma_bonus, int L,
-              int64_t d, int C4, uint64_t seed, const ChainState* __restrict__ state,
-              const float* __restrict__ part4, T* __restrict__ y) {
+              int64_t d, int C4, uint64_t seed_v, const uint64_t* __restrict__ seed_dev,
+              const ChainState* __restrict__ state, const float* __restrict__ part4, T* __restrict__ y) {
+  const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
   const ChainState cs = state[b];
   if (cs.kind == kKindInactive) return;
@@ -885,32 +971,60 @@ static void launch_verify(const VerifyArgs& A, int B, int L, int vpt, cudaStream
 }
 
 template <typename T>
+static void launch_tiles(const VerifyArgs& A, int B, int L, int vpt, cudaStream_t s) {
+  constexpr int V = 16 / (int)sizeof(T);
+  const bool vec = (A.d % V == 0) && aligned(A.x, 16) && aligned(A.mq, 16) && aligned(A.mp, 16);
+  const unsigned tiles = (unsigned)((int64_t)B * L * A.S.C);
+  if (!vec) {
+    k_tiles<T, false, 1><<<tiles, kK1Threads, 0, s>>>(A);
+    return;
+  }
+  switch (vpt) {
+    case 1: k_tiles<T, true, 1><<<tiles, kK1Threads, 0, s>>>(A); break;
+    case 2: k_tiles<T, true, 2><<<tiles, kK1Threads, 0, s>>>(A); break;
+    case 3: k_tiles<T, true, 3><<<tiles, kK1Threads, 0, s>>>(A); break;
+    default: k_tiles<T, true, 4><<<tiles, kK1Threads, 0, s>>>(A); break;
+  }
+}
+
+template <typename T, int RESID>
+static void launch_finish(const VerifyArgs& A, int B, cudaStream_t s) {
+  const bool vec4 = (A.d % 4 == 0) && aligned(A.x, 4 * sizeof(T)) && aligned(A.mq, 4 * sizeof(T)) &&
+                    aligned(A.mp, 4 * sizeof(T)) && (A.y == nullptr || aligned(A.y, 4 * sizeof(T))) &&
+                    (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
+  const int nt = RESID ? kFinishThreads : 32;
+  if (vec4) k_finish<T, true, RESID><<<B, nt, 0, s>>>(A);
+  else k_finish<T, false, RESID><<<B, nt, 0, s>>>(A);
+}
+
+template <typename T>
 static void launch_k4(const void* x, const void* mq, const void* mp, const void* mqb,
-                      const float* sb, int B, int L, int64_t d, uint64_t seed, const WsLayout& w,
+                      const float* sb, int B, int L, int64_t d, uint64_t seed, const uint64_t* seed_dev,
+                      const WsLayout& w,
                       const ChainState* st, float* part4, void* y, cudaStream_t s) {
   const bool vec = (d % 4 == 0) && aligned(x, 4 * sizeof(T)) && aligned(mq, 4 * sizeof(T)) &&
                    aligned(mp, 4 * sizeof(T)) && aligned(y, 4 * sizeof(T)) &&
                    (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
   const unsigned grid = (unsigned)((int64_t)B * w.C4);
   if (vec) {
-    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, st, part4);
+    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, seed_dev, st, part4);
     k_resid_write<T, true><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                      (const T*)mqb, sb, L, d, w.C4, seed, st, part4, (T*)y);
+                                                      (const T*)mqb, sb, L, d, w.C4, seed, seed_dev, st, part4, (T*)y);
   } else {
-    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, st, part4);
+    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, seed_dev, st, part4);
     k_resid_write<T, false><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                       (const T*)mqb, sb, L, d, w.C4, seed, st, part4, (T*)y);
+                                                       (const T*)mqb, sb, L, d, w.C4, seed, seed_dev, st, part4, (T*)y);
   }
 }
 
 // Enqueue the whole step (or, with ratios_only, the log-ratio pass) for validated args.
 static int enqueue_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
                           const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d,
-                          int dtype, uint64_t seed, int mode, const int32_t* L_eff,
+                          int dtype, uint64_t seed, const uint64_t* seed_dev, int mode, const int32_t* L_eff,
                           const void* mu_target_bonus, const float* sigma_bonus,
                           int residual_kind, float omega, int32_t* accepted_len, void* y_out,
                           float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
-                          float* chain_aux_out, bool ratios_only, void* workspace,
+                          float* chain_aux_out, bool ratios_only, bool timed, void* workspace,
                           cudaStream_t s) {
   const WsLayout w = ws_layout(B, L, d, dtype);
   char* ws = (char*)workspace;
@@ -923,39 +1037,88 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   ScanArgs& S = A.S;
   A.part = (float2*)(ws + w.part_off);
   S.part = A.part; S.C = w.C1; S.sigma = sigma; S.sstride = sigma_stride_b;
-  S.B = B; S.L = L; S.L_eff = L_eff; S.seed = seed; S.mode = mode;
+  S.B = B; S.L = L; S.L_eff = L_eff; S.seed = seed; S.seed_dev = seed_dev; S.mode = mode;
   S.inv_omega2 = 1.0f / (omega * omega); S.residual_kind = residual_kind;
   S.has_bonus = mu_target_bonus != nullptr; S.ratios_only = ratios_only; S.draw_u = true;
   S.ell_out = log_ratio_out; S.dn_out = delta_norm_out; S.accepted_len = accepted_len;
   S.status_out = status_out; S.aux_out = chain_aux_out;
 
-  cudaEvent_t* tev = ratios_only ? nullptr : timing_slot();
+  cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
-  if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
-    check_launch();
-    return SDV_ECUDA;
-  }
   const bool long_rows = (d + 3) / 4 > kFusedMaxGroups;
-  if (long_rows && !ratios_only) {
-    if (dtype == SDV_F32) launch_verify<float, 0>(A, B, L, w.vpt1, s);
-    else launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, s);
+  const bool many = !ratios_only && B >= kManyChainMin;
+  const bool f32 = dtype == SDV_F32;
+  if (many) {
+    if (f32) launch_tiles<float>(A, B, L, w.vpt1, s);
+    else launch_tiles<__nv_bfloat16>(A, B, L, w.vpt1, s);
   } else {
-    if (dtype == SDV_F32) launch_verify<float, 1>(A, B, L, w.vpt1, s);
-    else launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, s);
+    if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+      check_launch();
+      return SDV_ECUDA;
+    }
+    if (long_rows && !ratios_only) {
+      if (f32) launch_verify<float, 0>(A, B, L, w.vpt1, s);
+      else launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, s);
+    } else {
+      if (f32) launch_verify<float, 1>(A, B, L, w.vpt1, s);
+      else launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, s);
+    }
   }
   int rc = check_launch();
   if (rc != SDV_OK) return rc;
   if (tev) timing_record(tev[1], s);
+  if (many) {
+    if (long_rows) {
+      if (f32) launch_finish<float, 0>(A, B, s);
+      else launch_finish<__nv_bfloat16, 0>(A, B, s);
+    } else {
+      if (f32) launch_finish<float, 1>(A, B, s);
+      else launch_finish<__nv_bfloat16, 1>(A, B, s);
+    }
+    if ((rc = check_launch()) != SDV_OK) return rc;
+  }
   if (long_rows && !ratios_only) {
     float* part4 = (float*)(ws + w.part4_off);
-    if (dtype == SDV_F32)
-      launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, A.state, part4, y_out, s);
+    if (f32)
+      launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev, w, A.state, part4, y_out, s);
     else
-      launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, w, A.state, part4, y_out, s);
+      launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev, w, A.state, part4, y_out, s);
     rc = check_launch();
   }
   if (tev) timing_record(tev[2], s);
   return rc;
+}
+
+int verify_ex_impl(const void* x_draft, const void* mu_target, const void* mu_draft,
+                        const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                        uint64_t seed, const uint64_t* seed_dev, int mode, const int32_t* L_eff,
+                        const void* mu_target_bonus, const float* sigma_bonus, int residual_kind,
+                        float omega, int32_t* accepted_len, void* y_out, float* log_ratio_out,
+                        float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
+                        void* workspace, size_t workspace_bytes, bool timed, void* stream) {
+  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
+  if (rc != SDV_OK) return rc;
+  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
+  if (residual_kind != SDV_RESIDUAL_DECOMPOSITION && residual_kind != SDV_RESIDUAL_REFLECTION)
+    return SDV_EINVAL;
+  if (residual_kind == SDV_RESIDUAL_REFLECTION && mode != SDV_MODE_SAMPLE) return SDV_EINVAL;
+  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
+  if (!accepted_len || !y_out) return SDV_EINVAL;
+  if ((mu_target_bonus == nullptr) != (sigma_bonus == nullptr)) return SDV_EINVAL;
+  const size_t es = dtype == SDV_BF16 ? 2 : 4;
+  if (!aligned(y_out, es) || !aligned(accepted_len, 4) ||
+      (mu_target_bonus && !aligned(mu_target_bonus, es)) || (sigma_bonus && !aligned(sigma_bonus, 4)) ||
+      (L_eff && !aligned(L_eff, 4)) || (log_ratio_out && !aligned(log_ratio_out, 4)) ||
+      (delta_norm_out && !aligned(delta_norm_out, 4)) || (status_out && !aligned(status_out, 4)) ||
+      (chain_aux_out && !aligned(chain_aux_out, 4)) || (seed_dev && !aligned(seed_dev, 8)))
+    return SDV_EALIGN;
+  const WsLayout w = ws_layout(B, L, d, dtype);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if (!aligned(workspace, 256)) return SDV_EALIGN;
+  return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                        seed_dev, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+                        accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
+                        chain_aux_out, false, timed, workspace, (cudaStream_t)stream);
 }
 
 }  // namespace sdv
@@ -991,29 +1154,10 @@ int sdv_verify_ex(const void* x_draft, const void* mu_target, const void* mu_dra
                   int32_t* accepted_len, void* y_out, float* log_ratio_out,
                   float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
                   void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
-  int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
-  if (rc != SDV_OK) return rc;
-  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
-  if (residual_kind != SDV_RESIDUAL_DECOMPOSITION && residual_kind != SDV_RESIDUAL_REFLECTION)
-    return SDV_EINVAL;
-  if (residual_kind == SDV_RESIDUAL_REFLECTION && mode != SDV_MODE_SAMPLE) return SDV_EINVAL;
-  if (!(omega > 0.f) || !std::isfinite(omega)) return SDV_EINVAL;
-  if (!accepted_len || !y_out) return SDV_EINVAL;
-  if ((mu_target_bonus == nullptr) != (sigma_bonus == nullptr)) return SDV_EINVAL;
-  const size_t es = dtype == SDV_BF16 ? 2 : 4;
-  if (!aligned(y_out, es) || !aligned(accepted_len, 4) ||
-      (mu_target_bonus && !aligned(mu_target_bonus, es)) || (sigma_bonus && !aligned(sigma_bonus, 4)) ||
-      (L_eff && !aligned(L_eff, 4)) || (log_ratio_out && !aligned(log_ratio_out, 4)) ||
-      (delta_norm_out && !aligned(delta_norm_out, 4)) || (status_out && !aligned(status_out, 4)) ||
-      (chain_aux_out && !aligned(chain_aux_out, 4)))
-    return SDV_EALIGN;
-  const WsLayout w = ws_layout(B, L, d, dtype);
-  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
-  if (!aligned(workspace, 256)) return SDV_EALIGN;
-  return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
-                        mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+  return verify_ex_impl(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                        nullptr, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
                         accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
-                        chain_aux_out, false, workspace, (cudaStream_t)stream);
+                        chain_aux_out, workspace, workspace_bytes, true, stream);
 }
 
 int sdv_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
@@ -1040,9 +1184,9 @@ int sdv_log_ratios(const void* x_draft, const void* mu_target, const void* mu_dr
   if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
   if (!aligned(workspace, 256)) return SDV_EALIGN;
   return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, 0,
-                        SDV_MODE_BLOCK, L_eff, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION, 1.0f,
-                        nullptr, nullptr, log_ratio_out, delta_norm_out, nullptr, nullptr, true,
-                        workspace, (cudaStream_t)stream);
+                        nullptr, SDV_MODE_BLOCK, L_eff, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION,
+                        1.0f, nullptr, nullptr, log_ratio_out, delta_norm_out, nullptr, nullptr, true,
+                        false, workspace, (cudaStream_t)stream);
 }
 
 int sdv_accept_scan(const float* log_ratio, const float* delta_norm, int B, int L,

@@ -168,6 +168,42 @@ def test_verify_full_size_sampled(api, kind, sample, mode, m):
     compare(gs, o, m, inp["dtype"], max_tie_frac=0.1)
 
 
+# Many chains (B >= 512) take the two-kernel path: k_tiles streams, k_finish finishes
+# every chain with one warp (its own U-sampler and residual writer).
+@pytest.mark.parametrize("mode,m", MODES)
+@pytest.mark.parametrize("kind,B,L,d,sample", [("tiny", 600, 8, 64, None), ("latent", 520, 4, 1003, None),
+                                               ("pixel", 512, 3, 5000, 64), ("pixel", 1024, 16, 1024, 96)])
+def test_verify_many_chains_matches_oracle(api, mode, m, kind, B, L, d, sample):
+    inp = W.make_verify_inputs(kind, B=B, L=L, d=d)
+    g = run_gpu(api, inp, 4321, mode)
+    chains = np.arange(B) if sample is None else \
+        np.random.Generator(np.random.PCG64(6)).choice(B, sample, replace=False)
+    o = oracle_for(inp, 4321, m, chains=chains)
+    gs = {k: v[chains] for k, v in g.items()}
+    compare(gs, o, m, inp["dtype"])
+    both = np.isfinite(gs["aux"][:, 0]) & np.isfinite(o["U"]) & (gs["accepted_len"] == o["accepted_len"])
+    assert both.sum() > 0
+    assert np.all(np.abs(gs["aux"][both, 0] - o["U"][both]) <= 5e-6 + 3e-7 * np.abs(o["U"][both]))
+
+
+def test_verify_many_chains_ragged_bonus_reflection(api):
+    Bn = 640
+    inp = W.make_verify_inputs("pixel", B=Bn, L=6, d=300, per_chain_sigma=True)
+    rng = np.random.Generator(np.random.PCG64(18))
+    Leff = rng.integers(0, 7, Bn).astype(np.int32)
+    Leff[:3] = [0, 1, 6]
+    mqb = rng.standard_normal((Bn, 300)).astype(np.float32)
+    sb = rng.uniform(0.1, 1.0, Bn).astype(np.float32)
+    for mode, m in MODES:
+        g = run_gpu(api, inp, 78, mode, L_eff=Leff, mu_target_bonus=mqb, sigma_bonus=sb)
+        o = oracle_for(inp, 78, m, Leff=Leff, mu_target_bonus=mqb, sigma_bonus=sb)
+        assert np.all(g["accepted_len"][Leff == 0] == 0)
+        compare(g, o, m, "f32")
+    g = run_gpu(api, inp, 79, "sample", residual="reflection")
+    o = oracle_for(inp, 79, OV.MODE_SAMPLE, residual=OV.RESIDUAL_REFLECTION)
+    compare(g, o, OV.MODE_SAMPLE, "f32")
+
+
 def test_verify_ragged_windows_bonus_and_inactive(api):
     inp = W.make_verify_inputs("pixel", B=40, L=6, d=1000, per_chain_sigma=True)
     rng = np.random.Generator(np.random.PCG64(8))

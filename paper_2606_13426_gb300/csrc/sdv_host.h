@@ -20,7 +20,7 @@ constexpr int kK1MinBlocks = 3;
 // thread per residual sweep.
 constexpr int kManyChainMin = 512;
 constexpr int tile_min_blocks(int vpt) { return vpt <= 1 ? 8 : (vpt == 2 ? 6 : 4); }
-constexpr int kFinishThreads = 128;
+constexpr int kFinishThreads = 64;
 constexpr int kFinishResidUnroll = 4;
 // Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;

@@ -85,13 +85,14 @@ __device__ __forceinline__ void gmm_rows_warp(const GmmRow (&R)[RB], int nr, int
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int C = G.C;
-  float sab[RB], v[RB], be[RB];
+  float sab[RB], v[RB], inv_v[RB], be[RB];
 #pragma unroll
   for (int q = 0; q < RB; ++q) {
     const float tf = S.tfwd(R[q].k);
     const float ab = S.abar(tf);
     sab[q] = sqrtf(ab);
     v[q] = ab * G.comp_var + 1.0f - ab;
+    inv_v[q] = 1.0f / v[q];
     be[q] = S.beta(tf);
   }
   const float cst = 0.5f * (1.0f + S.churn * S.churn);
@@ -130,7 +131,8 @@ __device__ __forceinline__ void gmm_rows_warp(const GmmRow (&R)[RB], int nr, int
           if (q < nr) {
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const float df = (4 * gi + e < d) ? zf[q][e] - sab[q] * mf[e] : 0.f;
+              // the tail check is only needed without VEC (d % 4 == 0 otherwise)
+              const float df = (VEC || 4 * gi + e < d) ? zf[q][e] - sab[q] * mf[e] : 0.f;
               acc[q][c] = fmaf(df, df, acc[q][c]);
             }
           }
@@ -151,7 +153,7 @@ __device__ __forceinline__ void gmm_rows_warp(const GmmRow (&R)[RB], int nr, int
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) a += __shfl_xor_sync(FULL, a, o);
       }
-      acc[q][c] = (c < C) ? __ldg(G.log_w + c) - a / (2.0f * v[q]) : -INFINITY;
+      acc[q][c] = (c < C) ? __ldg(G.log_w + c) - 0.5f * a * inv_v[q] : -INFINITY;
       mx = fmaxf(mx, acc[q][c]);
     }
     float den = 0.f;
@@ -194,7 +196,7 @@ __device__ __forceinline__ void gmm_rows_warp(const GmmRow (&R)[RB], int nr, int
         float sc[4], m[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          sc[e] = (w_sc[q] * wsum[q][e] - zf[q][e]) / v[q];
+          sc[e] = (w_sc[q] * wsum[q][e] - zf[q][e]) * inv_v[q];
           m[e] = zf[q][e] + S.delta * (0.5f * be[q] * zf[q][e] + cst * be[q] * sc[e]) + R[q].add_sigma * G4[e];
         }
         float* score = R[q].score;
@@ -244,7 +246,7 @@ k_gmm_rows(const float* __restrict__ states, const int32_t* __restrict__ k, cons
 }
 
 // Rows of a round's parallel target call per warp.
-template <int MAXC> struct RoundRows { static constexpr int value = MAXC <= 8 ? 3 : 2; };
+template <int MAXC> struct RoundRows { static constexpr int value = MAXC <= 8 ? 3 : 1; };
 
 // Parallel target call of a round.  Row (b, j), j = 0 .. gamma_b, is state y[b]
 // (j = 0) or x_draft[b, j-1] at step k[b] + j; its mean goes to mu_target[b, j]

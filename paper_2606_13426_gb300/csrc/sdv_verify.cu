@@ -603,6 +603,7 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   __shared__ UParams P_s;
   __shared__ bool haveP_s;
   __shared__ USampleScratch us;
+  __shared__ float4 g_s[RESID ? kFusedMaxGroups : 1];  // the residual's G, drawn once
   const int L = A.S.L;
   const int C = A.S.C;
   const int64_t tile = blockIdx.x;
@@ -650,8 +651,8 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   if (RESID == 0) {
     if (threadIdx.x == 0) A.state[b] = cs;
   } else {
-    residual_row<T, VEC4, 1, false>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
-                                    b, cs, (T*)A.y, CtaGroup{red, &bcast}, nullptr);
+    residual_row<T, VEC4, 1, true>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
+                                   b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
   }
 }
 

@@ -295,6 +295,198 @@ k_round_target(const float* __restrict__ y, const float* __restrict__ x_draft,
   }
 }
 
+// Row slots of a round's target call, shared by the target-call kernels: slot
+// (b, j), j = 0 .. L, is live when j <= gamma_b (and gamma_b > 0).
+struct RoundRow {
+  const float* z;
+  float* mq;
+  float* score;
+  int k;
+  bool live;
+};
+
+__device__ __forceinline__ RoundRow round_row(int64_t slot, int64_t slots, const float* y, const float* x_draft,
+                                              const int32_t* kk, const int32_t* gam, int L, int64_t d,
+                                              const Sched& S, float* mu_target, float* mu_bonus,
+                                              float* sigma_bonus, float* sc_all, bool write_sigma) {
+  RoundRow R{nullptr, nullptr, nullptr, 0, false};
+  if (slot >= slots) return R;
+  const int b = (int)(slot / (L + 1));
+  const int j = (int)(slot - (int64_t)b * (L + 1));
+  const int g = gam[b];
+  if (j > g || g == 0) return R;
+  const int kb = kk[b];
+  R.z = (j == 0) ? y + (int64_t)b * d : x_draft + ((int64_t)b * L + j - 1) * d;
+  R.mq = (j < g) ? mu_target + ((int64_t)b * L + j) * d : mu_bonus + (int64_t)b * d;
+  R.score = sc_all + ((int64_t)b * (L + 1) + j) * d;
+  R.k = kb + j;
+  R.live = true;
+  if (j == g && write_sigma) sigma_bonus[b] = S.sigma(kb + g);
+  return R;
+}
+
+// Parallel target call of a round for rows of up to 4 kGmmThreads elements
+// (d % 4 == 0, 16-byte aligned rows): each thread owns one group of four elements
+// and holds that group of every mean in registers for the whole kernel; a CTA takes
+// RB = 32 / MAXC row slots at a time (grid-stride), keeps each row's group in
+// registers across both passes, and reduces the RB x MAXC squared distances with one
+// warp reduce-scatter (value v ends in lane v) and one pass over the warps.  Warp 0
+// resolves the next batch's rows and their schedule constants into shared memory
+// (three buffers: the batch being written, the one being finished and the next),
+// and every thread loads the next batch's states while this batch finishes.
+// Resident CTAs per SM k_round_target_reg is built for (its register budget).
+constexpr int round_reg_blocks(int maxc) { return maxc <= 8 ? 3 : 2; }
+
+template <int MAXC>
+__global__ void __launch_bounds__(kGmmThreads, round_reg_blocks(MAXC))
+k_round_target_reg(const float* __restrict__ y, const float* __restrict__ x_draft,
+                   const int32_t* __restrict__ kk, const int32_t* __restrict__ gam, int B, int L, int64_t d,
+                   Sched S, Gmm G, float* mu_target, float* mu_bonus, float* sigma_bonus, float* sc_all) {
+  constexpr int RB = 32 / MAXC;
+  constexpr int NV = RB * MAXC;  // 32
+  struct RowC {
+    const float* z;
+    float* mq;
+    float* score;
+    float sab, inv_v, be;
+    int live;
+  };
+  __shared__ float red[kGmmWarps][NV];
+  __shared__ float resp[RB][MAXC];
+  __shared__ float wsc[RB];
+  __shared__ RowC rows_s[3][RB];
+  const unsigned FULL = 0xffffffffu;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int C = G.C;
+  const int64_t ng = d / 4;
+  const bool own = tid < ng;  // this thread's group exists
+  const int64_t slots = (int64_t)B * (L + 1);
+  const int64_t stride = (int64_t)gridDim.x * RB;
+  // warp 0, lane r < RB: row slot s + r -> rows_s[buf][r]
+  auto resolve = [&](int64_t s, int buf) {
+    if (warp == 0 && lane < RB) {
+      const RoundRow R = round_row(s + lane, slots, y, x_draft, kk, gam, L, d, S, mu_target, mu_bonus,
+                                   sigma_bonus, sc_all, true);
+      RowC rc;
+      rc.z = R.z; rc.mq = R.mq; rc.score = R.score; rc.live = R.live ? 1 : 0;
+      const float tf = S.tfwd(R.k);
+      const float ab = S.abar(tf);
+      rc.sab = sqrtf(ab);
+      rc.inv_v = 1.0f / (ab * G.comp_var + 1.0f - ab);
+      rc.be = S.beta(tf);
+      rows_s[buf][lane] = rc;
+    }
+  };
+  float4 m4[MAXC];
+#pragma unroll
+  for (int c = 0; c < MAXC; ++c)
+    m4[c] = (own && c < C) ? __ldg(reinterpret_cast<const float4*>(G.means + (int64_t)c * d) + tid)
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float cst = 0.5f * (1.0f + S.churn * S.churn);
+  int64_t s0 = (int64_t)blockIdx.x * RB;
+  int cur = 0;
+  resolve(s0, cur);
+  __syncthreads();
+  float4 z[RB];
+#pragma unroll
+  for (int r = 0; r < RB; ++r)
+    z[r] = (rows_s[cur][r].live && own) ? *(reinterpret_cast<const float4*>(rows_s[cur][r].z) + tid)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+  for (; s0 < slots; s0 += stride) {
+    const int nxt = cur == 2 ? 0 : cur + 1;
+    const RowC* R = rows_s[cur];
+    // pass 1: this thread's share of |z_r - sqrt(abar_r) mu_c|^2
+    float v[NV];
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      const float zf[4] = {z[r].x, z[r].y, z[r].z, z[r].w};
+#pragma unroll
+      for (int c = 0; c < MAXC; ++c) {
+        const float mf[4] = {m4[c].x, m4[c].y, m4[c].z, m4[c].w};
+        float a = 0.f;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float df = zf[e] - R[r].sab * mf[e];
+          a = fmaf(df, df, a);
+        }
+        v[r * MAXC + c] = a;
+      }
+    }
+    // warp reduce-scatter: after the halving steps lane l holds the warp sum of value l
+#pragma unroll
+    for (int h = NV / 2; h >= 1; h >>= 1) {
+      const bool up = (lane & h) != 0;
+#pragma unroll
+      for (int k = 0; k < h; ++k) {
+        const float send = up ? v[k] : v[k + h];
+        const float keep = up ? v[k + h] : v[k];
+        v[k] = keep + __shfl_xor_sync(FULL, send, h);
+      }
+    }
+    red[warp][lane] = v[0];
+    resolve(s0 + stride, nxt);  // last read two batches ago, before this batch's first barrier
+    __syncthreads();
+    // the next batch's states, in flight while this batch finishes
+    float4 zn[RB];
+#pragma unroll
+    for (int r = 0; r < RB; ++r)
+      zn[r] = (rows_s[nxt][r].live && own) ? *(reinterpret_cast<const float4*>(rows_s[nxt][r].z) + tid)
+                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+    if (warp == 0) {
+      // responsibilities r_c = softmax(log w_c - d2_c / (2 v)) over each row's MAXC lanes
+      float t = 0.f;
+#pragma unroll
+      for (int w = 0; w < kGmmWarps; ++w) t += red[w][lane];
+      const int r = lane / MAXC, c = lane - r * MAXC;
+      float ivr = R[0].inv_v, sabr = R[0].sab;
+#pragma unroll
+      for (int q = 1; q < RB; ++q) {
+        ivr = (r == q) ? R[q].inv_v : ivr;
+        sabr = (r == q) ? R[q].sab : sabr;
+      }
+      const float a = (c < C) ? __ldg(G.log_w + c) - 0.5f * t * ivr : -INFINITY;
+      float mx = a;
+#pragma unroll
+      for (int o = MAXC / 2; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(FULL, mx, o));
+      const float ex = (c < C) ? expf(a - mx) : 0.f;
+      float den = ex;
+#pragma unroll
+      for (int o = MAXC / 2; o >= 1; o >>= 1) den += __shfl_xor_sync(FULL, den, o);
+      resp[r][c] = ex;
+      if (c == 0) wsc[r] = sabr / den;  // folds the softmax normaliser and sqrt(abar)
+    }
+    __syncthreads();
+    // pass 2: score and target mean of this thread's group
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      if (R[r].live && own) {
+        float ws[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < MAXC; ++c) {
+          const float rc = resp[r][c];
+          ws[0] = fmaf(rc, m4[c].x, ws[0]);
+          ws[1] = fmaf(rc, m4[c].y, ws[1]);
+          ws[2] = fmaf(rc, m4[c].z, ws[2]);
+          ws[3] = fmaf(rc, m4[c].w, ws[3]);
+        }
+        const float w = wsc[r];
+        const float zf[4] = {z[r].x, z[r].y, z[r].z, z[r].w};
+        float sc[4], m[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          sc[e] = (w * ws[e] - zf[e]) * R[r].inv_v;
+          m[e] = zf[e] + S.delta * (0.5f * R[r].be * zf[e] + cst * R[r].be * sc[e]);
+        }
+        reinterpret_cast<float4*>(R[r].score)[tid] = make_float4(sc[0], sc[1], sc[2], sc[3]);
+        reinterpret_cast<float4*>(R[r].mq)[tid] = make_float4(m[0], m[1], m[2], m[3]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) z[r] = zn[r];
+    cur = nxt;
+  }
+}
+
 // Free / Frozen drafter: gamma_b elementwise steps from y[b] with the cached score.
 // One thread per group of four elements; VEC: d % 4 == 0 and 16-byte aligned rows
 // (float4 loads and stores).  The Philox draws do not depend on the state, so the
@@ -501,6 +693,17 @@ static unsigned round_target_grid(const GmmLaunch& gl, int B, int L) {
   return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, 4 * (int64_t)sm_count()));
 }
 
+// Rows of up to 4 kGmmThreads elements with 16-byte aligned rows and means take the
+// register-resident k_round_target_reg (grid-stride over its resident CTAs); others
+// the shared-memory k_round_target.
+static bool round_target_reg(const GmmLaunch& gl, int64_t d) { return gl.vec && d <= 4 * kGmmThreads; }
+
+static unsigned round_target_reg_grid(const GmmLaunch& gl, int B, int L) {
+  const int64_t rb = 32 / (gl.maxc <= 8 ? 8 : 16);
+  const int64_t need = ((int64_t)B * (L + 1) + rb - 1) / rb;
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, round_reg_blocks(gl.maxc) * (int64_t)sm_count()));
+}
+
 #define SDV_GMM_DISPATCH(GL, KERNEL, GRID, STREAM, ...)                                          \
   do {                                                                                          \
     if ((GL).maxc == 8) {                                                                       \
@@ -696,8 +899,16 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
         rc = launch_check();
       }
       if (rc == SDV_OK) {
-        SDV_GMM_DISPATCH(gl, k_round_target, round_target_grid(gl, B, L), cs, y, xd, kk, gam, B, L, d, S, G,
-                         gl.smem, mqd, mqb, sgb, scall);
+        if (round_target_reg(gl, d)) {
+          const unsigned grid = round_target_reg_grid(gl, B, L);
+          if (gl.maxc == 8)
+            k_round_target_reg<8><<<grid, kGmmThreads, 0, cs>>>(y, xd, kk, gam, B, L, d, S, G, mqd, mqb, sgb, scall);
+          else
+            k_round_target_reg<16><<<grid, kGmmThreads, 0, cs>>>(y, xd, kk, gam, B, L, d, S, G, mqd, mqb, sgb, scall);
+        } else {
+          SDV_GMM_DISPATCH(gl, k_round_target, round_target_grid(gl, B, L), cs, y, xd, kk, gam, B, L, d, S, G,
+                           gl.smem, mqd, mqb, sgb, scall);
+        }
         rc = launch_check();
       }
       if (rc == SDV_OK)

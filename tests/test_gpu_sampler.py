@@ -90,13 +90,8 @@ def test_em_chain_matches_oracle(api):
     assert np.max(np.abs(y - yo) / np.maximum(1.0, np.abs(yo))) < 1e-4
 
 
-@pytest.mark.parametrize("mode", [OV.MODE_SAMPLE, OV.MODE_BLOCK])
-@pytest.mark.parametrize("drafter", ["free", "frozen"])
-def test_first_rounds_match_oracle(api, mode, drafter):
-    """Rounds 1..3 element by element: k, and the states of chains whose coins all lie
-    outside the tie band in every round so far."""
-    d, Bn, L, K = 64, 192, 4, 40
-    gmm = _gmm(8, d, 6)
+def _first_rounds(api, mode, drafter, d, C, Bn=192, L=4, K=40):
+    gmm = _gmm(C, d, 6)
     sch = OS.VPSchedule(K, 0.5)
     tgt = _target(api, gmm, K, 0.5)
     o = OS.speculative_sample(Bn, d, L, mode, gmm, sch, seed=123, drafter=drafter, max_rounds=3,
@@ -114,6 +109,21 @@ def test_first_rounds_match_oracle(api, mode, drafter):
         np.testing.assert_array_equal(k[clean], tr["k"][clean])
         err = np.abs(y[clean] - tr["y"][clean]) / np.maximum(1.0, np.abs(tr["y"][clean]))
         assert err.max() < 1e-4, err.max()
+
+
+@pytest.mark.parametrize("mode", [OV.MODE_SAMPLE, OV.MODE_BLOCK])
+@pytest.mark.parametrize("drafter", ["free", "frozen"])
+def test_first_rounds_match_oracle(api, mode, drafter):
+    """Rounds 1..3 element by element: k, and the states of chains whose coins all lie
+    outside the tie band in every round so far."""
+    _first_rounds(api, mode, drafter, 64, 8)
+
+
+# Row lengths and component counts that take the other target-call kernels: ragged d
+# and rows longer than 1024 elements (shared-memory means), 9..16 components.
+@pytest.mark.parametrize("d,C", [(37, 8), (1100, 8), (64, 12), (1024, 12), (1030, 12)])
+def test_first_rounds_other_shapes(api, d, C):
+    _first_rounds(api, OV.MODE_BLOCK, "free", d, C, Bn=96)
 
 
 def _check_law(y, m, var, n_sigma=4.0):

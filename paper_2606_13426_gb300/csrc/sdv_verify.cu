@@ -69,6 +69,13 @@ __device__ __forceinline__ void unpack(const uint4& v, float (&f)[8]) {
   }
 }
 
+// Ticket of a chain: fetch-and-add with acquire-release semantics at GPU scope.
+__device__ __forceinline__ unsigned int ticket_acq_rel(unsigned int* p) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
+  return old;
+}
+
 // Read-once streaming load: no L1 allocation.
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   uint4 r;
@@ -629,13 +636,13 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
   if (threadIdx.x == 0) {
     A.part[tile] = t;
-    __threadfence();  // publish the partial before taking the ticket
-    const unsigned int k = atomicAdd(A.ticket + b, 1u);
+    // release this partial with the ticket; the chain's last ticket also acquires
+    // every partial released before it (one acq_rel atomic instead of two fences)
+    const unsigned int k = ticket_acq_rel(A.ticket + b);
     last_s = (k == (unsigned int)(g * C) - 1u);
   }
-  __syncthreads();
+  __syncthreads();  // thread 0's acquire reaches warp 0's partial loads through the barrier
   if (!last_s) return;
-  __threadfence();  // acquire: every partial of chain b is visible
   if (threadIdx.x < 32) {
     const ScanOut so = scan_warp(A.S, b);
     if (threadIdx.x == 0) {

@@ -24,9 +24,14 @@ constexpr int kFinishThreads = 64;
 constexpr int kFinishResidUnroll = 4;
 // Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;
-// Long-row residual kernels: threads per CTA and elements of the rejected row per CTA.
+// Long-row residual kernels: threads per CTA, and the elements of the rejected row
+// per CTA, chosen per call between kK4MinChunk and kK4MaxChunk so that the grid is
+// about kK4TargetCtas CTAs (short kernels want many CTAs; long rows want fewer,
+// longer ones).
 constexpr int kK4Threads = 256;
-constexpr int kK4Chunk = 4096;
+constexpr int64_t kK4MinChunk = 1024;
+constexpr int64_t kK4MaxChunk = 4096;
+constexpr int64_t kK4TargetCtas = 1024;
 // Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
 // finishes the chain inside the fused kernel; longer rows by k_resid_dot/_write.
 constexpr int64_t kFusedMaxGroups = 1024;
@@ -85,6 +90,7 @@ struct WsLayout {
   int vpt1;        // K1 16-byte vectors per thread per tensor
   int64_t chunk1;  // elements of a row per K1 tile
   int C1;          // K1 tiles per row
+  int64_t chunk4;  // K4 elements per tile
   int C4;          // K4 tiles per chain
   size_t ticket_off, part_off, state_off, part4_off, total;
 };

@@ -732,7 +732,7 @@ __global__ void __launch_bounds__(kK2Threads) k_scan(ScanArgs A) {
 // ---------------------------------------------------------------- long rows: K4a / K4b
 template <typename T, bool VEC4>
 __global__ void __launch_bounds__(kK4Threads)
-k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d, int C4,
+k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d, int C4, int gpc,
             uint64_t seed_v, const uint64_t* __restrict__ seed_dev, const ChainState* __restrict__ state,
             float* __restrict__ part4) {
   __shared__ float2 red[kK4Threads / 32];
@@ -741,8 +741,8 @@ k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d
   const ChainState cs = state[b];
   if (cs.kind != kKindResid) return;
   const int64_t base = ((int64_t)b * L + cs.row) * d;
-  const int64_t g0 = (int64_t)c * (kK4Chunk / 4);
-  const int64_t g1 = min(g0 + kK4Chunk / 4, (d + 3) / 4);
+  const int64_t g0 = (int64_t)c * gpc;
+  const int64_t g1 = min(g0 + gpc, (d + 3) / 4);
   float s = 0.f;
   for (int64_t gi = g0 + threadIdx.x; gi < g1; gi += kK4Threads) {
     float fq[4], fp[4];
@@ -762,7 +762,7 @@ template <typename T, bool VEC4>
 __global__ void __launch_bounds__(kK4Threads)
 k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __restrict__ mp,
               const T* __restrict__ mq_bonus, const float* __restrict__ sigma_bonus, int L,
-              int64_t d, int C4, uint64_t seed_v, const uint64_t* __restrict__ seed_dev,
+              int64_t d, int C4, int gpc, uint64_t seed_v, const uint64_t* __restrict__ seed_dev,
               const ChainState* __restrict__ state, const float* __restrict__ part4, T* __restrict__ y) {
   const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
@@ -770,8 +770,8 @@ k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __rest
   if (cs.kind == kKindInactive) return;
   const int64_t rbase = ((int64_t)b * L + cs.row) * d;
   const int64_t ybase = (int64_t)b * d;
-  const int64_t g0 = (int64_t)c * (kK4Chunk / 4);
-  const int64_t g1 = min(g0 + kK4Chunk / 4, (d + 3) / 4);
+  const int64_t g0 = (int64_t)c * gpc;
+  const int64_t g1 = min(g0 + gpc, (d + 3) / 4);
   float coef = 0.f;  // U - e^T G for the decomposition residual
   if (cs.kind == kKindResid) {
     float T2 = 0.f;
@@ -918,7 +918,12 @@ WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   w.vpt1 = (int)std::min<int64_t>(kK1Vpt, std::max<int64_t>(1, (vec_per_row + kK1Threads - 1) / kK1Threads));
   w.chunk1 = (int64_t)kK1Threads * w.vpt1 * (16 / es);
   w.C1 = (int)((d + w.chunk1 - 1) / w.chunk1);
-  w.C4 = (int)((d + kK4Chunk - 1) / kK4Chunk);
+  // long-row residual chunks: about kK4TargetCtas CTAs over all chains, kK4MinChunk ..
+  // kK4MaxChunk elements each (a power of two)
+  int64_t chunk4 = kK4MinChunk;
+  while (chunk4 < kK4MaxChunk && (int64_t)B * ((d + chunk4 - 1) / chunk4) > kK4TargetCtas) chunk4 *= 2;
+  w.chunk4 = chunk4;
+  w.C4 = (int)((d + chunk4 - 1) / chunk4);
   auto up = [](size_t v) { return (v + 255) & ~(size_t)255; };
   size_t off = 0;
   w.ticket_off = off;
@@ -1015,13 +1020,13 @@ static void launch_k4(const void* x, const void* mq, const void* mp, const void*
                    (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
   const unsigned grid = (unsigned)((int64_t)B * w.C4);
   if (vec) {
-    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, seed_dev, st, part4);
+    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4);
     k_resid_write<T, true><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                      (const T*)mqb, sb, L, d, w.C4, seed, seed_dev, st, part4, (T*)y);
+                                                      (const T*)mqb, sb, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4, (T*)y);
   } else {
-    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, seed, seed_dev, st, part4);
+    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4);
     k_resid_write<T, false><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                       (const T*)mqb, sb, L, d, w.C4, seed, seed_dev, st, part4, (T*)y);
+                                                       (const T*)mqb, sb, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4, (T*)y);
   }
 }
 

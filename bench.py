@@ -49,6 +49,10 @@ def parse():
     p.add_argument("--workload", default="pixel", choices=["pixel", "latent", "highres", "sampler"])
     p.add_argument("--sampler-L", default="4,8,16",
                    help="draft windows of the end-to-end sampler workload")
+    p.add_argument("--sampler-rounds", type=int, default=0,
+                   help="sampler workload only: instead of the timed runs, drive this many "
+                        "rounds from the host (sdv_sampler_begin / _round / _end, block mode), "
+                        "twice per window, so that a profiler sees every kernel launch")
     p.add_argument("--mode", default="block", choices=["block", "sample"])
     p.add_argument("--batch", type=int, default=0,
                    help="chains per call (0: the workload's B); smaller batches serve ncu captures")
@@ -236,6 +240,34 @@ def run_reference(args, world, rank):
     print(json.dumps(line))
 
 
+def run_sampler_rounds(args, rank, local):
+    """Host-driven sampler rounds (profiling aid): per window L, two runs of
+    begin + R rounds + end in block mode; prints the time per round of the second."""
+    import torch
+    import __graft_entry__ as G
+    G.build()
+    from paper_2606_13426_gb300 import api
+    torch.cuda.set_device(local)
+    cfg = W.SAMPLER_CONFIG
+    gm = W.make_gmm()
+    tgt = api.GmmTarget(torch.from_numpy(gm["means"]), torch.from_numpy(gm["log_weights"]),
+                        gm["comp_var"], cfg["K"], cfg["churn"])
+    Bn, d, R = cfg["B"], cfg["d"], args.sampler_rounds
+    runs = {}
+    for L in [int(v) for v in args.sampler_L.split(",")]:
+        ws = torch.empty(api.B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8, device="cuda")
+        for _ in range(2):
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            r = api.sampler_rounds(Bn, L, tgt, 100, R, "block", workspace=ws)
+            torch.cuda.synchronize()
+            t = time.perf_counter() - t0
+        runs["L%d_block" % L] = {"rounds": r["rounds"], "us_per_round": 1e6 * t / max(1, R)}
+    if rank == 0:
+        print(json.dumps({"metric": "host-driven sampler rounds (profiling aid, not a bench value)",
+                          "config": {"B": Bn, "d": d, "rounds": R}, "runs": runs}))
+
+
 def run_sampler(args, world, rank, local):
     """End-to-end speculative sampler on the analytic 8-component mixture (B = 1024 chains,
     d = 1024, K = 1000 VP Euler-Maruyama steps, churn 0.5, Free drafter) against the plain
@@ -296,6 +328,9 @@ def main():
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.workload == "sampler" and args.sampler_rounds > 0:
+        run_sampler_rounds(args, rank, local)
         return
     if args.workload == "sampler":
         run_sampler(args, world, rank, local)

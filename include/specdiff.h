@@ -303,6 +303,31 @@ int sdv_sampler_run(int B, int L, int64_t d, const float *means, const float *lo
                     size_t workspace_bytes, sdv_stream_t stream);
 
 /*
+ * Host-driven rounds: the same sampler as sdv_sampler_run, one call per round.
+ * sdv_sampler_begin draws Y_0 and makes the initial target call (the chains'
+ * bookkeeping and round state live in the workspace); each sdv_sampler_round
+ * enqueues one round (the same kernels, in the same order, as one iteration of
+ * sdv_sampler_run's graph, so that begin + R rounds + end gives the same results
+ * as sdv_sampler_run with max_rounds = R while a chain is active; a round with no
+ * active chain only advances the round counter); sdv_sampler_end synchronises
+ * `stream` and returns the same outputs as sdv_sampler_run.  Every round must pass
+ * the arguments given to begin (and one mode and drafter throughout).  All three
+ * return SDV_EINVAL / SDV_ENOWORKSPACE / SDV_EALIGN for bad arguments as
+ * sdv_sampler_run does, before launching anything.
+ */
+int sdv_sampler_begin(int B, int L, int64_t d, const float *means, const float *log_weights, int C,
+                      float comp_var, int K, float churn, float beta_min, float beta_max,
+                      float t_floor, uint64_t seed, void *workspace, size_t workspace_bytes,
+                      sdv_stream_t stream);
+int sdv_sampler_round(int B, int L, int64_t d, const float *means, const float *log_weights, int C,
+                      float comp_var, int K, float churn, float beta_min, float beta_max,
+                      float t_floor, uint64_t seed, int mode, int drafter, void *workspace,
+                      size_t workspace_bytes, sdv_stream_t stream);
+int sdv_sampler_end(int B, int L, int64_t d, void *workspace, size_t workspace_bytes, float *y_out,
+                    int32_t *k_out, int32_t *chain_rounds_out, int32_t *tau_sum_out,
+                    int32_t *rounds_out, sdv_stream_t stream);
+
+/*
  * sdv_em_sample - the plain (non-speculative) Euler-Maruyama chain, Y_{k+1} =
  * m^q_k(Y_k) + sigma_k G_k for k = 0 .. K-1 from Y_0 (stream 5), G_k from stream 6 with
  * sub-counter k; y_out [B, d] fp32 out.  K kernel launches on `stream`.

@@ -248,6 +248,28 @@ def sampler_run(Bn, L, target, seed, mode="block", drafter="free", max_rounds=No
     return dict(y=y, k=k, chain_rounds=cr, tau_sum=ts, rounds=rounds)
 
 
+def sampler_rounds(Bn, L, target, seed, rounds, mode="block", drafter="free", workspace=None):
+    """The same sampler driven from the host: sdv_sampler_begin, `rounds` calls of
+    sdv_sampler_round, sdv_sampler_end; returns the dict of sampler_run."""
+    dev = target.means.device
+    d = target.d
+    if workspace is None:
+        workspace = torch.empty(B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8,
+                                device=dev)
+    y = torch.empty(Bn, d, dtype=torch.float32, device=dev)
+    k = torch.empty(Bn, dtype=torch.int32, device=dev)
+    cr = torch.empty(Bn, dtype=torch.int32, device=dev)
+    ts = torch.empty(Bn, dtype=torch.int32, device=dev)
+    dr = {"free": B.SDV_DRAFTER_FREE, "frozen": B.SDV_DRAFTER_FROZEN}[drafter]
+    sd = int(seed) & 0xFFFFFFFFFFFFFFFF
+    ws, nb, st = _ptr(workspace), workspace.numel(), _stream()
+    B.sdv_sampler_begin(Bn, L, d, *target.params(), sd, ws, nb, st)
+    for _ in range(int(rounds)):
+        B.sdv_sampler_round(Bn, L, d, *target.params(), sd, _MODES[mode], dr, ws, nb, st)
+    r = B.sdv_sampler_end(Bn, L, d, ws, nb, _ptr(y), _ptr(k), _ptr(cr), _ptr(ts), st)
+    return dict(y=y, k=k, chain_rounds=cr, tau_sum=ts, rounds=r)
+
+
 def em_sample(Bn, target, seed):
     """The plain Euler-Maruyama chain (sdv_em_sample)."""
     y = torch.empty(Bn, target.d, dtype=torch.float32, device=target.means.device)

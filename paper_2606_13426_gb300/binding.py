@@ -64,6 +64,10 @@ SIGNATURES = {
     "sdv_sampler_workspace_bytes": (_SZ, [_I, _I, _I64]),
     "sdv_sampler_run": (_I, [_I, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _I, _I, _I,
                              _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "sdv_sampler_begin": (_I, [_I, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _P, _SZ, _P]),
+    "sdv_sampler_round": (_I, [_I, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _I, _I, _P,
+                               _SZ, _P]),
+    "sdv_sampler_end": (_I, [_I, _I, _I64, _P, _SZ, _P, _P, _P, _P, _P, _P]),
     "sdv_em_sample": (_I, [_I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _U64, _P, _P]),
     "sdv_timing_enable": (_I, [_I]),
     "sdv_timing_stride": (_I, [_I]),
@@ -218,6 +222,27 @@ def sdv_sampler_run(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min
     _call("sdv_sampler_run", B, L, d, means, log_weights, C, comp_var, K, churn, beta_min,
           beta_max, t_floor, seed, mode, drafter, max_rounds, y_out, k_out, chain_rounds_out,
           tau_sum_out, ctypes.addressof(rounds), workspace, workspace_bytes, stream)
+    return int(rounds.value)
+
+
+def sdv_sampler_begin(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max,
+                      t_floor, seed, workspace, workspace_bytes, stream):
+    return _call("sdv_sampler_begin", B, L, d, means, log_weights, C, comp_var, K, churn, beta_min,
+                 beta_max, t_floor, seed, workspace, workspace_bytes, stream)
+
+
+def sdv_sampler_round(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max,
+                      t_floor, seed, mode, drafter, workspace, workspace_bytes, stream):
+    return _call("sdv_sampler_round", B, L, d, means, log_weights, C, comp_var, K, churn, beta_min,
+                 beta_max, t_floor, seed, mode, drafter, workspace, workspace_bytes, stream)
+
+
+def sdv_sampler_end(B, L, d, workspace, workspace_bytes, y_out, k_out, chain_rounds_out,
+                    tau_sum_out, stream):
+    """Returns the number of rounds run (the C call's rounds_out)."""
+    rounds = ctypes.c_int32(0)
+    _call("sdv_sampler_end", B, L, d, workspace, workspace_bytes, y_out, k_out, chain_rounds_out,
+          tau_sum_out, ctypes.addressof(rounds), stream)
     return int(rounds.value)
 
 

@@ -590,15 +590,17 @@ struct SamplerCtl {
   uint32_t active;
 };
 
-// End of a round (one thread): advance the round counter and seed, and keep the loop
-// of the round graph going while a chain is active and fewer than max_rounds ran.
-__global__ void k_round_close(SamplerCtl* ctl, uint64_t seed, int max_rounds, cudaGraphConditionalHandle h) {
+// End of a round (one thread): advance the round counter and seed, and (inside the
+// round graph) keep the loop going while a chain is active and fewer than
+// max_rounds rounds ran.
+__global__ void k_round_close(SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
+                              cudaGraphConditionalHandle h) {
   const int r = ctl->r + 1;
   ctl->r = r;
   ctl->seed_r = round_seed(seed, r);
   const bool more = ctl->active != 0u && r < max_rounds;
   ctl->active = 0u;
-  cudaGraphSetConditional(h, more ? 1u : 0u);
+  if (in_loop) cudaGraphSetConditional(h, more ? 1u : 0u);
 }
 
 __global__ void __launch_bounds__(256)
@@ -767,6 +769,139 @@ static SamplerLayout sampler_layout(int B, int L, int64_t d) {
   return w;
 }
 
+// A sampler problem and the views of its workspace.
+struct SamplerRun {
+  int B, L;
+  int64_t d;
+  int K, mode, drafter;
+  uint64_t seed;
+  Sched S;
+  Gmm G;
+  GmmLaunch gl;
+  unsigned eg;
+  float *y, *sc, *xd, *mpd, *mqd, *mqb, *sg, *sgb, *scall, *yo;
+  int32_t *kk, *gam, *acc, *rounds, *tsum;
+  SamplerCtl* ctl;
+  void* vws;
+  size_t vws_bytes;
+};
+
+static void sampler_views(const SamplerLayout& w, char* ws, SamplerRun* R) {
+  R->y = (float*)(ws + w.y);
+  R->sc = (float*)(ws + w.s);
+  R->kk = (int32_t*)(ws + w.k);
+  R->gam = (int32_t*)(ws + w.g);
+  R->xd = (float*)(ws + w.x);
+  R->mpd = (float*)(ws + w.mp);
+  R->mqd = (float*)(ws + w.mq);
+  R->mqb = (float*)(ws + w.mqb);
+  R->sg = (float*)(ws + w.sg);
+  R->sgb = (float*)(ws + w.sgb);
+  R->scall = (float*)(ws + w.sc);
+  R->acc = (int32_t*)(ws + w.acc);
+  R->yo = (float*)(ws + w.yo);
+  R->rounds = (int32_t*)(ws + w.rounds);
+  R->tsum = (int32_t*)(ws + w.tausum);
+  R->ctl = (SamplerCtl*)(ws + w.ctl);
+  R->vws = ws + w.vws;
+  R->vws_bytes = w.total - w.vws;
+}
+
+static int sampler_setup(int B, int L, int64_t d, const float* means, const float* log_weights, int C,
+                         float comp_var, int K, float churn, float beta_min, float beta_max, float t_floor,
+                         uint64_t seed, int mode, int drafter, void* workspace, size_t workspace_bytes,
+                         SamplerRun* R) {
+  if (!means || !log_weights) return SDV_EINVAL;
+  if (B < 1 || L < 1 || L > SDV_MAX_L || d < 1 || C < 1 || C > kSdvMaxComponents) return SDV_EINVAL;
+  if (!(comp_var > 0.f) || !valid_sched(K, churn, beta_min, beta_max, t_floor)) return SDV_EINVAL;
+  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
+  if (drafter != SDV_DRAFTER_FREE && drafter != SDV_DRAFTER_FROZEN) return SDV_EINVAL;
+  const SamplerLayout w = sampler_layout(B, L, d);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SDV_EALIGN;
+  R->B = B; R->L = L; R->d = d; R->K = K; R->mode = mode; R->drafter = drafter; R->seed = seed;
+  R->S = make_sched(K, churn, beta_min, beta_max, t_floor);
+  R->G = Gmm{means, log_weights, C, comp_var};
+  // workspace arrays start on 256-byte boundaries
+  R->gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(workspace) % 16 == 0);
+  R->eg = (unsigned)(((int64_t)B * ((d + 3) / 4) + 255) / 256);
+  sampler_views(w, (char*)workspace, R);
+  return SDV_OK;
+}
+
+// Initial states, bookkeeping and round state, and the only explicit target call: the
+// score at Y_0 (step 0).
+static int enqueue_begin(const SamplerRun& R, cudaStream_t s) {
+  k_sampler_init<<<R.eg, 256, 0, s>>>(R.B, R.L, R.d, R.K, R.seed, R.y, R.kk, R.gam, R.rounds, R.tsum, R.ctl);
+  int rc = launch_check();
+  if (rc != SDV_OK) return rc;
+  SDV_GMM_DISPATCH(R.gl, k_gmm_rows, rows_grid(R.B), s, R.y, R.kk, nullptr, R.B, R.d, R.S, R.G, R.gl.smem,
+                   nullptr, R.sc);
+  return launch_check();
+}
+
+// One round on stream cs (captured into the round graph's loop body when `loop`,
+// whose condition k_round_close then sets; launched directly otherwise).
+static int enqueue_round(const SamplerRun& R, cudaStream_t cs, int max_rounds, bool loop,
+                         cudaGraphConditionalHandle handle) {
+  const int B = R.B, L = R.L;
+  const int64_t d = R.d;
+  const GmmLaunch& gl = R.gl;
+  int rc = SDV_OK;
+  if (R.drafter == SDV_DRAFTER_FROZEN) {  // a fresh score at the round's start state
+    SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), cs, R.y, R.kk, R.gam, B, d, R.S, R.G, gl.smem, nullptr, R.sc);
+    if ((rc = launch_check()) != SDV_OK) return rc;
+  }
+  if (gl.vec)
+    k_draft<true><<<R.eg, 256, 0, cs>>>(R.y, R.sc, R.kk, R.gam, B, L, d, R.S, 0, &R.ctl->seed_r, R.xd, R.mpd, R.sg);
+  else
+    k_draft<false><<<R.eg, 256, 0, cs>>>(R.y, R.sc, R.kk, R.gam, B, L, d, R.S, 0, &R.ctl->seed_r, R.xd, R.mpd, R.sg);
+  if ((rc = launch_check()) != SDV_OK) return rc;
+  if (round_target_reg(gl, d)) {
+    const unsigned grid = round_target_reg_grid(gl, B, L);
+    if (gl.maxc == 8)
+      k_round_target_reg<8><<<grid, kGmmThreads, 0, cs>>>(R.y, R.xd, R.kk, R.gam, B, L, d, R.S, R.G, R.mqd, R.mqb,
+                                                         R.sgb, R.scall);
+    else
+      k_round_target_reg<16><<<grid, kGmmThreads, 0, cs>>>(R.y, R.xd, R.kk, R.gam, B, L, d, R.S, R.G, R.mqd, R.mqb,
+                                                          R.sgb, R.scall);
+  } else {
+    SDV_GMM_DISPATCH(gl, k_round_target, round_target_grid(gl, B, L), cs, R.y, R.xd, R.kk, R.gam, B, L, d, R.S,
+                     R.G, gl.smem, R.mqd, R.mqb, R.sgb, R.scall);
+  }
+  if ((rc = launch_check()) != SDV_OK) return rc;
+  rc = verify_ex_impl(R.xd, R.mqd, R.mpd, R.sg, L, B, L, d, SDV_F32, 0, &R.ctl->seed_r, R.mode, R.gam, R.mqb,
+                      R.sgb, SDV_RESIDUAL_DECOMPOSITION, 1.0f, R.acc, R.yo, nullptr, nullptr, nullptr, nullptr,
+                      R.vws, R.vws_bytes, false, cs);
+  if (rc != SDV_OK) return rc;
+  k_round_update<<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam, R.rounds,
+                                    R.tsum, &R.ctl->active);
+  if ((rc = launch_check()) != SDV_OK) return rc;
+  k_round_close<<<1, 1, 0, cs>>>(R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
+  return launch_check();
+}
+
+// Rounds run (host, after a synchronisation) and the chains' outputs (device copies).
+static int read_results(const SamplerRun& R, float* y_out, int32_t* k_out, int32_t* chain_rounds_out,
+                        int32_t* tau_sum_out, int32_t* rounds_out, cudaStream_t s) {
+  const int B = R.B;
+  int r = 0;
+  if (cudaMemcpyAsync(&r, &R.ctl->r, sizeof(r), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
+  *rounds_out = r;
+  if (cudaMemcpyAsync(y_out, R.y, (size_t)B * R.d * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
+  if (k_out && cudaMemcpyAsync(k_out, R.kk, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
+  if (chain_rounds_out &&
+      cudaMemcpyAsync(chain_rounds_out, R.rounds, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
+  if (tau_sum_out && cudaMemcpyAsync(tau_sum_out, R.tsum, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    return launch_check(), SDV_ECUDA;
+  return SDV_OK;
+}
+
 }  // namespace sdv
 
 using namespace sdv;
@@ -821,48 +956,14 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
                     float* y_out, int32_t* k_out, int32_t* chain_rounds_out,
                     int32_t* tau_sum_out, int32_t* rounds_out, void* workspace,
                     size_t workspace_bytes, sdv_stream_t stream) {
-  if (!means || !log_weights || !y_out || !rounds_out) return SDV_EINVAL;
-  if (B < 1 || L < 1 || L > SDV_MAX_L || d < 1 || C < 1 || C > kSdvMaxComponents) return SDV_EINVAL;
-  if (!(comp_var > 0.f) || !valid_sched(K, churn, beta_min, beta_max, t_floor)) return SDV_EINVAL;
-  if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
-  if (drafter != SDV_DRAFTER_FREE && drafter != SDV_DRAFTER_FROZEN) return SDV_EINVAL;
+  if (!y_out || !rounds_out) return SDV_EINVAL;
   if (max_rounds < 0) return SDV_EINVAL;
-  const SamplerLayout w = sampler_layout(B, L, d);
-  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
-  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SDV_EALIGN;
+  SamplerRun R;
+  int rc = sampler_setup(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max, t_floor, seed,
+                         mode, drafter, workspace, workspace_bytes, &R);
+  if (rc != SDV_OK) return rc;
   cudaStream_t s = (cudaStream_t)stream;
-  char* ws = (char*)workspace;
-  float* y = (float*)(ws + w.y);
-  float* sc = (float*)(ws + w.s);
-  int32_t* kk = (int32_t*)(ws + w.k);
-  int32_t* gam = (int32_t*)(ws + w.g);
-  float* xd = (float*)(ws + w.x);
-  float* mpd = (float*)(ws + w.mp);
-  float* mqd = (float*)(ws + w.mq);
-  float* mqb = (float*)(ws + w.mqb);
-  float* sg = (float*)(ws + w.sg);
-  float* sgb = (float*)(ws + w.sgb);
-  float* scall = (float*)(ws + w.sc);
-  int32_t* acc = (int32_t*)(ws + w.acc);
-  float* yo = (float*)(ws + w.yo);
-  int32_t* rounds = (int32_t*)(ws + w.rounds);
-  int32_t* tsum = (int32_t*)(ws + w.tausum);
-  SamplerCtl* ctl = (SamplerCtl*)(ws + w.ctl);
-  void* vws = ws + w.vws;
-  const size_t vws_bytes = w.total - w.vws;
-  const Sched S = make_sched(K, churn, beta_min, beta_max, t_floor);
-  const Gmm G{means, log_weights, C, comp_var};
-  const int64_t ng = (int64_t)B * ((d + 3) / 4);
-  const unsigned eg = (unsigned)((ng + 255) / 256);
-  // workspace arrays start on 256-byte boundaries
-  const GmmLaunch gl = gmm_launch(C, d, means, reinterpret_cast<uintptr_t>(workspace) % 16 == 0);
-
-  int rc;
-  k_sampler_init<<<eg, 256, 0, s>>>(B, L, d, K, seed, y, kk, gam, rounds, tsum, ctl);
-  if ((rc = launch_check()) != SDV_OK) return rc;
-  // the only explicit target call: the score at Y_0 (step 0)
-  SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), s, y, kk, nullptr, B, d, S, G, gl.smem, nullptr, sc);
-  if ((rc = launch_check()) != SDV_OK) return rc;
+  if ((rc = enqueue_begin(R, s)) != SDV_OK) return rc;
 
   // The round loop is one CUDA graph: a while node whose body is one round, captured
   // once; the round's seed lives in device memory (SamplerCtl) and k_round_close ends
@@ -888,41 +989,7 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
          cudaStreamBeginCaptureToGraph(cs, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal) ==
              cudaSuccess;
     if (ok) {
-      rc = SDV_OK;
-      if (drafter == SDV_DRAFTER_FROZEN) {  // a fresh score at the round's start state
-        SDV_GMM_DISPATCH(gl, k_gmm_rows, rows_grid(B), cs, y, kk, gam, B, d, S, G, gl.smem, nullptr, sc);
-        rc = launch_check();
-      }
-      if (rc == SDV_OK) {
-        if (gl.vec) k_draft<true><<<eg, 256, 0, cs>>>(y, sc, kk, gam, B, L, d, S, 0, &ctl->seed_r, xd, mpd, sg);
-        else k_draft<false><<<eg, 256, 0, cs>>>(y, sc, kk, gam, B, L, d, S, 0, &ctl->seed_r, xd, mpd, sg);
-        rc = launch_check();
-      }
-      if (rc == SDV_OK) {
-        if (round_target_reg(gl, d)) {
-          const unsigned grid = round_target_reg_grid(gl, B, L);
-          if (gl.maxc == 8)
-            k_round_target_reg<8><<<grid, kGmmThreads, 0, cs>>>(y, xd, kk, gam, B, L, d, S, G, mqd, mqb, sgb, scall);
-          else
-            k_round_target_reg<16><<<grid, kGmmThreads, 0, cs>>>(y, xd, kk, gam, B, L, d, S, G, mqd, mqb, sgb, scall);
-        } else {
-          SDV_GMM_DISPATCH(gl, k_round_target, round_target_grid(gl, B, L), cs, y, xd, kk, gam, B, L, d, S, G,
-                           gl.smem, mqd, mqb, sgb, scall);
-        }
-        rc = launch_check();
-      }
-      if (rc == SDV_OK)
-        rc = verify_ex_impl(xd, mqd, mpd, sg, L, B, L, d, SDV_F32, 0, &ctl->seed_r, mode, gam, mqb, sgb,
-                            SDV_RESIDUAL_DECOMPOSITION, 1.0f, acc, yo, nullptr, nullptr, nullptr, nullptr,
-                            vws, vws_bytes, false, cs);
-      if (rc == SDV_OK) {
-        k_round_update<<<B, 256, 0, cs>>>(acc, yo, xd, scall, L, d, K, y, sc, kk, gam, rounds, tsum, &ctl->active);
-        rc = launch_check();
-      }
-      if (rc == SDV_OK) {
-        k_round_close<<<1, 1, 0, cs>>>(ctl, seed, max_rounds, handle);
-        rc = launch_check();
-      }
+      rc = enqueue_round(R, cs, max_rounds, true, handle);
       cudaGraph_t captured = nullptr;
       const bool ended = cudaStreamEndCapture(cs, &captured) == cudaSuccess;
       ok = rc == SDV_OK && ended && cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess &&
@@ -936,21 +1003,42 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
       return launch_check(), SDV_ECUDA;
     }
   }
-  int r = 0;
-  if (cudaMemcpyAsync(&r, &ctl->r, sizeof(r), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
-      cudaStreamSynchronize(s) != cudaSuccess)
-    return launch_check(), SDV_ECUDA;
-  *rounds_out = r;
-  if (cudaMemcpyAsync(y_out, y, (size_t)B * d * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    return launch_check(), SDV_ECUDA;
-  if (k_out && cudaMemcpyAsync(k_out, kk, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    return launch_check(), SDV_ECUDA;
-  if (chain_rounds_out &&
-      cudaMemcpyAsync(chain_rounds_out, rounds, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    return launch_check(), SDV_ECUDA;
-  if (tau_sum_out && cudaMemcpyAsync(tau_sum_out, tsum, (size_t)B * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    return launch_check(), SDV_ECUDA;
-  return SDV_OK;
+  return read_results(R, y_out, k_out, chain_rounds_out, tau_sum_out, rounds_out, s);
+}
+
+int sdv_sampler_begin(int B, int L, int64_t d, const float* means, const float* log_weights, int C,
+                      float comp_var, int K, float churn, float beta_min, float beta_max, float t_floor,
+                      uint64_t seed, void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  SamplerRun R;
+  const int rc = sampler_setup(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max, t_floor,
+                               seed, SDV_MODE_BLOCK, SDV_DRAFTER_FREE, workspace, workspace_bytes, &R);
+  if (rc != SDV_OK) return rc;
+  return enqueue_begin(R, (cudaStream_t)stream);
+}
+
+int sdv_sampler_round(int B, int L, int64_t d, const float* means, const float* log_weights, int C,
+                      float comp_var, int K, float churn, float beta_min, float beta_max, float t_floor,
+                      uint64_t seed, int mode, int drafter, void* workspace, size_t workspace_bytes,
+                      sdv_stream_t stream) {
+  SamplerRun R;
+  const int rc = sampler_setup(B, L, d, means, log_weights, C, comp_var, K, churn, beta_min, beta_max, t_floor,
+                               seed, mode, drafter, workspace, workspace_bytes, &R);
+  if (rc != SDV_OK) return rc;
+  return enqueue_round(R, (cudaStream_t)stream, 0, false, 0);
+}
+
+int sdv_sampler_end(int B, int L, int64_t d, void* workspace, size_t workspace_bytes, float* y_out,
+                    int32_t* k_out, int32_t* chain_rounds_out, int32_t* tau_sum_out, int32_t* rounds_out,
+                    sdv_stream_t stream) {
+  if (!y_out || !rounds_out) return SDV_EINVAL;
+  if (B < 1 || L < 1 || L > SDV_MAX_L || d < 1) return SDV_EINVAL;
+  const SamplerLayout w = sampler_layout(B, L, d);
+  if (!workspace || workspace_bytes < w.total) return SDV_ENOWORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return SDV_EALIGN;
+  SamplerRun R{};
+  R.B = B; R.L = L; R.d = d;
+  sampler_views(w, (char*)workspace, &R);
+  return read_results(R, y_out, k_out, chain_rounds_out, tau_sum_out, rounds_out, (cudaStream_t)stream);
 }
 
 int sdv_em_sample(int B, int64_t d, const float* means, const float* log_weights, int C,

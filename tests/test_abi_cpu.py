@@ -88,6 +88,41 @@ def test_host_validation_rejects_before_launch(lib):
     assert lib.sdv_normals(0, 0, 16, 2, 0, 0x100, None) == B.SDV_EINVAL
 
 
+def test_sampler_entry_points_validate_before_launch(lib):
+    from paper_2606_13426_gb300 import binding as B
+    sch = (8, 1.0, 40, 0.5, 0.1, 20.0, 1e-4)       # C, comp_var, K, churn, beta_min, beta_max, t_floor
+    wsb = B.sdv_sampler_workspace_bytes(4, 4, 16)
+    assert wsb > 0 and B.sdv_sampler_workspace_bytes(4, 65, 16) == 0
+
+    def begin(**kw):
+        a = dict(B=4, L=4, d=16, means=0x1000, lw=0x2000, ws=0x100000, wsb=wsb)
+        a.update(kw)
+        return lib.sdv_sampler_begin(a["B"], a["L"], a["d"], a["means"], a["lw"], *sch, 1, a["ws"],
+                                     a["wsb"], None)
+
+    def rnd(**kw):
+        a = dict(B=4, L=4, d=16, mode=1, drafter=0, ws=0x100000, wsb=wsb)
+        a.update(kw)
+        return lib.sdv_sampler_round(a["B"], a["L"], a["d"], 0x1000, 0x2000, *sch, 1, a["mode"],
+                                     a["drafter"], a["ws"], a["wsb"], None)
+
+    assert begin(means=0) == B.SDV_EINVAL
+    assert begin(B=0) == B.SDV_EINVAL
+    assert begin(L=65) == B.SDV_EINVAL
+    assert begin(ws=0) == B.SDV_ENOWORKSPACE
+    assert begin(wsb=wsb - 1) == B.SDV_ENOWORKSPACE
+    assert begin(ws=0x100010) == B.SDV_EALIGN
+    assert rnd(mode=2) == B.SDV_EINVAL
+    assert rnd(drafter=5) == B.SDV_EINVAL
+    assert rnd(ws=0) == B.SDV_ENOWORKSPACE
+    y = ctypes.c_int32(0)
+    assert lib.sdv_sampler_end(4, 4, 16, 0x100000, wsb, 0, 0, 0, 0, ctypes.addressof(y), None) == B.SDV_EINVAL
+    assert lib.sdv_sampler_end(4, 4, 16, 0, wsb, 0x3000, 0, 0, 0, ctypes.addressof(y), None) == \
+        B.SDV_ENOWORKSPACE
+    assert lib.sdv_sampler_end(0, 4, 16, 0x100000, wsb, 0x3000, 0, 0, 0, ctypes.addressof(y), None) == \
+        B.SDV_EINVAL
+
+
 def test_python_binding_raises_on_error(lib):
     from paper_2606_13426_gb300 import binding as B
     with pytest.raises(B.SDVError) as ei:

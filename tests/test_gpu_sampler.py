@@ -119,6 +119,20 @@ def test_first_rounds_match_oracle(api, mode, drafter):
     _first_rounds(api, mode, drafter, 64, 8)
 
 
+@pytest.mark.parametrize("mode,drafter", [("block", "free"), ("sample", "frozen")])
+def test_host_driven_rounds_equal_graph_run(api, mode, drafter):
+    """begin + R rounds + end launches the kernels of R iterations of the round graph:
+    identical outputs, bit for bit."""
+    d, Bn, L, K = 64, 160, 4, 40
+    tgt = _target(api, _gmm(8, d, 11), K, 0.5)
+    for R in (1, 5):
+        g = api.sampler_run(Bn, L, tgt, 77, mode, drafter, max_rounds=R)
+        h = api.sampler_rounds(Bn, L, tgt, 77, R, mode, drafter)
+        assert g["rounds"] == h["rounds"] == R
+        for key in ("y", "k", "chain_rounds", "tau_sum"):
+            assert torch.equal(g[key], h[key]), key
+
+
 # Row lengths and component counts that take the other target-call kernels: ragged d
 # and rows longer than 1024 elements (shared-memory means), 9..16 components.
 @pytest.mark.parametrize("d,C", [(37, 8), (1100, 8), (64, 12), (1024, 12), (1030, 12)])

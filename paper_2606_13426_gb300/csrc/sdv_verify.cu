@@ -487,9 +487,11 @@ struct CtaGroup {
 // the group calls it with the same cs).  Decomposition: pass A reduces delta^T G,
 // pass B writes m^q + sigma (G + e (U - e^T G)).  With gcache (room for the row's
 // groups, used only by the thread that owns a group) pass A keeps G there for pass
-// B (GCACHE); without it pass B draws G again (same Philox counters).  Each thread handles RU
+// B (GMODE 1), or the caller has filled it already (GMODE 2: drawn by warps that
+// would otherwise wait on the scan); with GMODE 0 pass B draws G again (same
+// Philox counters).  Each thread handles RU
 // groups of four elements per sweep, the loads of all of them issued before any use.
-template <typename T, bool VEC4, int RU, bool GCACHE, typename Group>
+template <typename T, bool VEC4, int RU, int GMODE, typename Group>
 __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
                              const T* __restrict__ mp, const T* __restrict__ mq_bonus,
                              const float* __restrict__ sigma_bonus, int L, int64_t d,
@@ -513,8 +515,9 @@ __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
 #pragma unroll
       for (int u = 0; u < RU; ++u) {
         const int64_t gi = g0 + (int64_t)u * nt;
-        const float4 G = normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-        if (GCACHE && gi < ng) gcache[gi] = G;
+        const float4 G = (GMODE == 2) ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
+                                      : normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+        if (GMODE == 1 && gi < ng) gcache[gi] = G;
         sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
         sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
         sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
@@ -532,7 +535,7 @@ __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
 #pragma unroll
       for (int u = 0; u < RU; ++u) {
         const int64_t gi = g0 + (int64_t)u * nt;
-        const float4 G = GCACHE ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
+        const float4 G = GMODE ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
                                 : normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
         const float g4[4] = {G.x, G.y, G.z, G.w};
         float out[4];
@@ -582,6 +585,14 @@ __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
       if (gi < ng) store4<T, VEC4>(y + ybase, 4 * gi, d, out);
     }
   }
+}
+
+// The residual's G of chain b (stream kStreamResid) for groups [first, ng), every
+// `step`-th group, into gcache: drawn by the finishing CTA's warps other than the
+// scanning warp, before the rejected step is known (G does not depend on it).
+__device__ __forceinline__ void prefill_resid_g(uint64_t seed, int b, int64_t ng, int first, int step,
+                                                float4* gcache) {
+  for (int64_t gi = first; gi < ng; gi += step) gcache[gi] = normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
 }
 
 // ---------------------------------------------------------------- the fused kernel
@@ -650,6 +661,8 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
       P_s = so.P;
       haveP_s = so.have_P;
     }
+  } else if (RESID && !A.S.ratios_only) {
+    prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, kK1Threads - 32, g_s);
   }
   __syncthreads();
   if (A.S.ratios_only) return;
@@ -658,8 +671,8 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   if (RESID == 0) {
     if (threadIdx.x == 0) A.state[b] = cs;
   } else {
-    residual_row<T, VEC4, 1, true>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
-                                   b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
+    residual_row<T, VEC4, 1, 2>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
+                                b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
   }
 }
 
@@ -688,9 +701,10 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   if (threadIdx.x == 0) A.part[tile] = t;
 }
 
-// One CTA per chain: warp 0 scans the chain and draws U (warp U-sampler); then, with
-// RESID = 1, all kFinishThreads threads write y (launched with 32 threads and
-// leaving the chain state for k_resid_* when RESID = 0).
+// One CTA per chain: warp 0 scans the chain and draws U (warp U-sampler) while the
+// other warps draw the residual's G into shared memory; then, with RESID = 1, all
+// kFinishThreads threads write y (launched with 32 threads and leaving the chain
+// state for k_resid_* when RESID = 0).
 template <typename T, bool VEC4, int RESID>
 __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
   __shared__ ChainState cs_s;
@@ -713,11 +727,13 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
       if (RESID == 0) A.state[b] = cs;
       else cs_s = cs;
     }
+  } else if (RESID) {
+    prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, kFinishThreads - 32, g_s);
   }
   if (RESID == 0) return;
   __syncthreads();
   const ChainState cs = cs_s;
-  residual_row<T, VEC4, kFinishResidUnroll, true>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
+  residual_row<T, VEC4, kFinishResidUnroll, 2>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
                                             (const T*)A.mq_bonus, A.sigma_bonus, A.S.L, A.d, seed_of(A.S),
                                             b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
 }

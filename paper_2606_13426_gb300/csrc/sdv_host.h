@@ -13,7 +13,7 @@ constexpr int kK1Threads = 256;
 constexpr int kK1Vpt = 4;
 // Resident CTAs per SM the fused kernel is built for (its register budget): the
 // chain-finishing code needs more than the streaming loop.
-constexpr int kK1MinBlocks = 3;
+constexpr int kK1MinBlocks = 4;
 // Many-chain path (B >= kManyChainMin): resident CTAs per SM of the streaming
 // kernel k_tiles (its register budget: 3 x vpt 16-byte buffers per thread), and
 // the finishing kernel k_finish: threads per chain and groups of four elements per

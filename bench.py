@@ -201,6 +201,11 @@ def cpu_oracle_rate(inp, seed, mode, seconds, max_chains=None):
     return chains_done * L / t_total, chains_done, t_total
 
 
+def workload_name(args, Bn, L, d, dt_name):
+    """config.workload of a verify run, identical in both arms."""
+    return "%s verify (B=%d, L=%d, d=%d %s), %s mode" % (args.workload, Bn, L, d, dt_name, args.mode)
+
+
 def run_reference(args, world, rank):
     """Reference arm: the CPU oracle as it stands, on the host cores, same workload/metric."""
     if rank != 0:
@@ -231,7 +236,9 @@ def run_reference(args, world, rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": "%s verify, %s mode" % (W.describe(args.workload), args.mode)},
+        "config": {"workload": workload_name(args, cfg["B"], cfg["L"], cfg["d"], cfg["dtype"]),
+                   "global_batch": cfg["B"], "window": cfg["L"], "dim": cfg["d"],
+                   "parallelism": "host, one thread"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": "%d chain(s) of the %s batch per step (oracle.verify, numpy fp64)"
                                    % (per_step, args.workload)},
@@ -493,8 +500,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32" if dt_name == "f32" else "bf16",
         "data": "synthetic",
-        "config": {"workload": "%s verify (B=%d, L=%d, d=%d %s), %s mode"
-                               % (args.workload, Bn, L, d, dt_name, args.mode),
+        "config": {"workload": workload_name(args, Bn, L, d, dt_name),
                    "global_batch": world * Bn, "window": L, "dim": d,
                    "parallelism": "replicas" if world > 1 else "single-gpu",
                    "l2": "%d rotating input sets, %.0f MB > L2 %.0f MB" % (

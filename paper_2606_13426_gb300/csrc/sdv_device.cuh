@@ -481,6 +481,16 @@ __device__ __forceinline__ float usample_warp(const UParams& P, uint32_t wbits, 
   return ue + step;
 }
 
+// ---------------------------------------------------------------- tickets
+// Fetch-and-add of 1 with acquire-release semantics at GPU scope: the release
+// publishes this thread's earlier writes, and the holder of the last ticket
+// acquires every write released before it.
+__device__ __forceinline__ unsigned int ticket_acq_rel(unsigned int* p) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
+  return old;
+}
+
 // ---------------------------------------------------------------- element access
 template <typename T> struct Elem;
 template <> struct Elem<float> {

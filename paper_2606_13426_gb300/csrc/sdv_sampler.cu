@@ -551,56 +551,77 @@ k_draft(const float* __restrict__ y, const float* __restrict__ s_cache, const in
   }
 }
 
-// Round bookkeeping, one CTA per chain: the emitted state, the score cache, k, the next
-// window length and the statistics; counts the chains that remain active.
-__global__ void __launch_bounds__(256)
-k_round_update(const int32_t* __restrict__ acc, const float* __restrict__ y_out,
-               const float* __restrict__ x_draft, const float* __restrict__ sc_all, int L, int64_t d,
-               int K, float* y, float* s_cache, int32_t* kk, int32_t* gam, int32_t* rounds,
-               int32_t* tau_sum, unsigned int* active) {
-  const int b = blockIdx.x;
-  const int g = gam[b];
-  const int k = kk[b];
-  __syncthreads();  // every thread has read k and gamma before thread 0 updates them
-  if (g == 0) return;
-  const int tau = acc[b] + 1;
-  const bool end = (tau == g + 1) && (k + g >= K);  // no bonus step past the end of sampling
-  const float* ysrc = end ? x_draft + ((int64_t)b * L + g - 1) * d : y_out + (int64_t)b * d;
-  const float* ssrc = sc_all + ((int64_t)b * (L + 1) + min(tau, g)) * d;
-  for (int64_t i = threadIdx.x; i < d; i += blockDim.x) {
-    y[(int64_t)b * d + i] = ysrc[i];
-    s_cache[(int64_t)b * d + i] = ssrc[i];
-  }
-  if (threadIdx.x == 0) {
-    const int kn = min(k + tau, K);
-    kk[b] = kn;
-    const int gn = kn < K ? min(L, K - kn) : 0;
-    gam[b] = gn;
-    rounds[b] += 1;
-    tau_sum[b] += tau;
-    if (gn > 0) atomicAdd(active, 1u);
-  }
-}
-
 // Device-resident state of the round loop: the seed of the current round, the rounds
 // run, and the chains k_round_update found still active in the current round.
 struct SamplerCtl {
   uint64_t seed_r;
   int32_t r;
   uint32_t active;
+  uint32_t done;  // chains whose update finished this round
 };
 
-// End of a round (one thread): advance the round counter and seed, and (inside the
-// round graph) keep the loop going while a chain is active and fewer than
-// max_rounds rounds ran.
-__global__ void k_round_close(SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
-                              cudaGraphConditionalHandle h) {
+// End of a round (the last chain's CTA, after every chain's ticket): advance the
+// round counter and seed, reset the round's counters, and (inside the round graph)
+// keep the loop going while a chain is active and fewer than max_rounds rounds ran.
+__device__ __forceinline__ void close_round(SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
+                                            cudaGraphConditionalHandle h) {
   const int r = ctl->r + 1;
   ctl->r = r;
   ctl->seed_r = round_seed(seed, r);
   const bool more = ctl->active != 0u && r < max_rounds;
   ctl->active = 0u;
+  ctl->done = 0u;
   if (in_loop) cudaGraphSetConditional(h, more ? 1u : 0u);
+}
+
+// Round bookkeeping, one CTA per chain: the emitted state, the score cache, k, the next
+// window length and the statistics; counts the chains that remain active, and the
+// CTA holding the round's last ticket closes the round (close_round).
+// VEC: d % 4 == 0 (workspace rows are then 16-byte aligned).
+template <bool VEC>
+__global__ void __launch_bounds__(256)
+k_round_update(const int32_t* __restrict__ acc, const float* __restrict__ y_out,
+               const float* __restrict__ x_draft, const float* __restrict__ sc_all, int L, int64_t d,
+               int K, float* y, float* s_cache, int32_t* kk, int32_t* gam, int32_t* rounds,
+               int32_t* tau_sum, SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
+               cudaGraphConditionalHandle h) {
+  const int b = blockIdx.x;
+  const int g = gam[b];
+  const int k = kk[b];
+  __syncthreads();  // every thread has read k and gamma before thread 0 updates them
+  const int tau = acc[b] + 1;
+  if (g > 0) {
+    const bool end = (tau == g + 1) && (k + g >= K);  // no bonus step past the end of sampling
+    const float* ysrc = end ? x_draft + ((int64_t)b * L + g - 1) * d : y_out + (int64_t)b * d;
+    const float* ssrc = sc_all + ((int64_t)b * (L + 1) + min(tau, g)) * d;
+    if (VEC) {
+      const float4* ys4 = reinterpret_cast<const float4*>(ysrc);
+      const float4* ss4 = reinterpret_cast<const float4*>(ssrc);
+      float4* yd4 = reinterpret_cast<float4*>(y + (int64_t)b * d);
+      float4* sd4 = reinterpret_cast<float4*>(s_cache + (int64_t)b * d);
+      for (int64_t i = threadIdx.x; i < d / 4; i += blockDim.x) {
+        yd4[i] = ys4[i];
+        sd4[i] = ss4[i];
+      }
+    } else {
+      for (int64_t i = threadIdx.x; i < d; i += blockDim.x) {
+        y[(int64_t)b * d + i] = ysrc[i];
+        s_cache[(int64_t)b * d + i] = ssrc[i];
+      }
+    }
+  }
+  if (threadIdx.x == 0) {
+    if (g > 0) {
+      const int kn = min(k + tau, K);
+      kk[b] = kn;
+      const int gn = kn < K ? min(L, K - kn) : 0;
+      gam[b] = gn;
+      rounds[b] += 1;
+      tau_sum[b] += tau;
+      if (gn > 0) atomicAdd(&ctl->active, 1u);
+    }
+    if (ticket_acq_rel(&ctl->done) == gridDim.x - 1) close_round(ctl, seed, max_rounds, in_loop, h);
+  }
 }
 
 __global__ void __launch_bounds__(256)
@@ -620,6 +641,7 @@ k_sampler_init(int B, int L, int64_t d, int K, uint64_t seed, float* y, int32_t*
     ctl->seed_r = round_seed(seed, 0);
     ctl->r = 0;
     ctl->active = 0u;
+    ctl->done = 0u;
   }
   if (gi == 0 && kk != nullptr) {
     kk[b] = 0;
@@ -841,7 +863,8 @@ static int enqueue_begin(const SamplerRun& R, cudaStream_t s) {
 }
 
 // One round on stream cs (captured into the round graph's loop body when `loop`,
-// whose condition k_round_close then sets; launched directly otherwise).
+// whose condition the round's last update CTA then sets; launched directly
+// otherwise).
 static int enqueue_round(const SamplerRun& R, cudaStream_t cs, int max_rounds, bool loop,
                          cudaGraphConditionalHandle handle) {
   const int B = R.B, L = R.L;
@@ -874,10 +897,12 @@ static int enqueue_round(const SamplerRun& R, cudaStream_t cs, int max_rounds, b
                       R.sgb, SDV_RESIDUAL_DECOMPOSITION, 1.0f, R.acc, R.yo, nullptr, nullptr, nullptr, nullptr,
                       R.vws, R.vws_bytes, false, cs);
   if (rc != SDV_OK) return rc;
-  k_round_update<<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam, R.rounds,
-                                    R.tsum, &R.ctl->active);
-  if ((rc = launch_check()) != SDV_OK) return rc;
-  k_round_close<<<1, 1, 0, cs>>>(R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
+  if (d % 4 == 0)
+    k_round_update<true><<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam,
+                                            R.rounds, R.tsum, R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
+  else
+    k_round_update<false><<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam,
+                                             R.rounds, R.tsum, R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
   return launch_check();
 }
 
@@ -966,8 +991,8 @@ int sdv_sampler_run(int B, int L, int64_t d, const float* means, const float* lo
   if ((rc = enqueue_begin(R, s)) != SDV_OK) return rc;
 
   // The round loop is one CUDA graph: a while node whose body is one round, captured
-  // once; the round's seed lives in device memory (SamplerCtl) and k_round_close ends
-  // the loop.  One graph launch runs every round with no host round trip.
+  // once; the round's seed lives in device memory (SamplerCtl) and the round's last
+  // update CTA ends the loop.  One graph launch runs every round with no host round trip.
   if (max_rounds > 0) {
     cudaGraph_t graph = nullptr, body = nullptr;
     cudaGraphExec_t exec = nullptr;

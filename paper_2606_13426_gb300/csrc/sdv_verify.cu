@@ -69,13 +69,6 @@ __device__ __forceinline__ void unpack(const uint4& v, float (&f)[8]) {
   }
 }
 
-// Ticket of a chain: fetch-and-add with acquire-release semantics at GPU scope.
-__device__ __forceinline__ unsigned int ticket_acq_rel(unsigned int* p) {
-  unsigned int old;
-  asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(p) : "memory");
-  return old;
-}
-
 // Read-once streaming load: no L1 allocation.
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   uint4 r;

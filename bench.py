@@ -175,6 +175,27 @@ def fused_kernel_bytes(B, L, d, dtype):
     return main if (long_rows(d) or many_chains(B)) else main + 3 * B * d * s
 
 
+def input_seed(base, i, rank):
+    """Seed of input set i on this rank: every rank verifies its own chains (weak scaling,
+    no data-path collective)."""
+    return base + 100 * i + 7 * rank
+
+
+def max_over_ranks(x, pg, device):
+    """The largest of the ranks' values of x (the job's time is its slowest rank's)."""
+    if pg is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, units_per_rank, seconds):
+    """Units processed by all ranks per second of the slowest rank."""
+    return world * units_per_rank / seconds
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -374,7 +395,7 @@ def main():
     sets = []
     host0 = None
     for i in range(n_sets):
-        inp = W.make_verify_inputs(args.workload, B=Bn, seed=cfg["seed"] + 100 * i + 7 * rank)
+        inp = W.make_verify_inputs(args.workload, B=Bn, seed=input_seed(cfg["seed"], i, rank))
         sets.append(dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"),
                          mp=to_dev(inp, "mu_draft"), sigma=torch.from_numpy(inp["sigma"]).to(dev)))
         if i == 0:
@@ -448,13 +469,11 @@ def main():
     n_timed = max(1, -(-last_len // TIMING_STRIDE))
     kv_ms, kr_ms, _ = (v / n_timed for v in binding.sdv_timing_read(n_timed))
     binding.sdv_timing_enable(0)
+    ms_total = max_over_ranks(ms_total, pg, dev)
     if pg:
-        t = torch.tensor([ms_total], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms_total = float(t.item())
         pg.barrier()
     ms_step = ms_total / args.steps
-    value = world * Bn * L / (ms_step * 1e-3)
+    value = whole_job_rate(world, Bn * L, ms_step * 1e-3)
 
     # mean tau per target call, block and sample, over the input sets
     taus = {}

@@ -222,6 +222,41 @@ def cpu_oracle_rate(inp, seed, mode, seconds, max_chains=None):
     return chains_done * L / t_total, chains_done, t_total
 
 
+def _oracle_worker(job):
+    """One process of the all-cores oracle timing: the same input set, its own chains."""
+    workload, Bn, seed, mode, seconds, wid, nw, barrier = job
+    from oracle import verify as OV
+    inp = W.make_verify_inputs(workload, B=Bn, seed=seed)
+    m = OV.MODE_BLOCK if mode == "block" else OV.MODE_SAMPLE
+    own = np.arange(wid, Bn, nw)
+    barrier.wait()
+    chains_done, t_total, calls = 0, 0.0, 0
+    while t_total < seconds:
+        t0 = time.perf_counter()
+        OV.verify(inp["x_draft"], inp["mu_target"], inp["mu_draft"], inp["sigma"], 1000 * wid + calls,
+                  m, chains=own)
+        t_total += time.perf_counter() - t0
+        chains_done += len(own)
+        calls += 1
+    return chains_done, t_total
+
+
+def cpu_oracle_rate_all_cores(workload, Bn, seed, mode, seconds, nproc):
+    """The oracle as it stands in nproc spawned processes (one thread each), each on its
+    own share of the chains of the same input set, started together."""
+    import multiprocessing as mpl
+    ctx = mpl.get_context("spawn")
+    with ctx.Manager() as mgr:
+        barrier = mgr.Barrier(nproc)
+        with ctx.Pool(nproc) as pool:
+            res = pool.map(_oracle_worker, [(workload, Bn, seed, mode, seconds, w, nproc, barrier)
+                                            for w in range(nproc)])
+    chains = sum(r[0] for r in res)
+    t = max(r[1] for r in res)
+    L = W.VERIFY_CONFIGS[workload]["L"]
+    return chains * L / t, chains, t
+
+
 def workload_name(args, Bn, L, d, dt_name):
     """config.workload of a verify run, identical in both arms."""
     return "%s verify (B=%d, L=%d, d=%d %s), %s mode" % (args.workload, Bn, L, d, dt_name, args.mode)
@@ -298,8 +333,9 @@ def run_sampler_rounds(args, rank, local):
 
 def run_sampler(args, world, rank, local):
     """End-to-end speculative sampler on the analytic 8-component mixture (B = 1024 chains,
-    d = 1024, K = 1000 VP Euler-Maruyama steps, churn 0.5, Free drafter) against the plain
-    Euler-Maruyama chain: wall-clock, rounds and accepted steps per parallel target call."""
+    d = 1024, K = 1000 VP Euler-Maruyama steps, churn 0.5, Free and Frozen drafters)
+    against the plain Euler-Maruyama chain: wall-clock, rounds and accepted steps per
+    parallel target call (the Frozen drafter makes one more target call per round)."""
     import torch
     import __graft_entry__ as G
     G.build()
@@ -323,28 +359,30 @@ def run_sampler(args, world, rank, local):
     runs = {}
     for L in [int(v) for v in args.sampler_L.split(",")]:
         ws = torch.empty(api.B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8, device="cuda")
-        for mode in ("sample", "block"):
-            timed(lambda: api.sampler_run(Bn, L, tgt, 7, mode, workspace=ws))
-            best = None
-            for i in range(3):
-                r, t = timed(lambda: api.sampler_run(Bn, L, tgt, 100 + i, mode, workspace=ws))
-                if best is None or t < best[1]:
-                    best = (r, t)
-            r, t = best
-            cr = r["chain_rounds"].cpu().numpy().astype(np.float64)
-            ts = r["tau_sum"].cpu().numpy().astype(np.float64)
-            runs["L%d_%s" % (L, mode)] = {
-                "ms": 1e3 * t, "rounds": r["rounds"], "mean_chain_rounds": float(cr.mean()),
-                "mean_tau": float(ts.sum() / cr.sum()),
-                "target_calls_per_chain": float(cr.mean() + 1.0),
-                "speedup_vs_em": t_em / t}
+        for drafter in ("free", "frozen"):
+            for mode in ("sample", "block"):
+                timed(lambda: api.sampler_run(Bn, L, tgt, 7, mode, drafter, workspace=ws))
+                best = None
+                for i in range(3):
+                    r, t = timed(lambda: api.sampler_run(Bn, L, tgt, 100 + i, mode, drafter, workspace=ws))
+                    if best is None or t < best[1]:
+                        best = (r, t)
+                r, t = best
+                cr = r["chain_rounds"].cpu().numpy().astype(np.float64)
+                ts = r["tau_sum"].cpu().numpy().astype(np.float64)
+                calls_per_round = 2.0 if drafter == "frozen" else 1.0
+                runs["L%d_%s%s" % (L, mode, "_frozen" if drafter == "frozen" else "")] = {
+                    "ms": 1e3 * t, "rounds": r["rounds"], "mean_chain_rounds": float(cr.mean()),
+                    "mean_tau": float(ts.sum() / cr.sum()),
+                    "target_calls_per_chain": float(calls_per_round * cr.mean() + 1.0),
+                    "speedup_vs_em": t_em / t}
     best_key = min(runs, key=lambda k2: runs[k2]["ms"])
     line = {
         "metric": "end-to-end speculative sampler: denoising steps/s; mean accepted steps/target call",
         "value": Bn * K / (runs[best_key]["ms"] * 1e-3), "unit": "denoising steps/s",
         "n_gpus": 1, "higher_is_better": True, "dtype": "f32", "data": "synthetic",
         "config": {"workload": "analytic 8-component GMM, d=%d, B=%d, K=%d VP EM steps, churn %.2f, "
-                               "Free drafter" % (d, Bn, K, cfg["churn"]), "best": best_key},
+                               "Free and Frozen drafters" % (d, Bn, K, cfg["churn"]), "best": best_key},
         "em_ms": 1e3 * t_em, "em_steps_per_s": Bn * K / t_em, "runs": runs,
     }
     if rank == 0:
@@ -550,6 +588,14 @@ def main():
                                 "sample": "%d chains of the %s batch through oracle.verify "
                                           "(numpy fp64, one thread), %.1f s"
                                           % (nch, args.workload, tsec)}
+        if Bn == cfg["B"]:
+            nproc = max(1, min(os.cpu_count() or 1, Bn))
+            prate, pch, pt = cpu_oracle_rate_all_cores(args.workload, Bn, input_seed(cfg["seed"], 0, 0),
+                                                       args.mode, args.cpu_seconds, nproc)
+            line["cpu_baseline_all_cores"] = {
+                "value": prate, "unit": UNIT, "cores": nproc, "kind": "oracle",
+                "sample": "%d chains of the %s batch through oracle.verify (numpy fp64) in %d "
+                          "spawned processes of one thread, %.1f s each" % (pch, args.workload, nproc, pt)}
     if rank == 0:
         print(json.dumps(line))
     if pg:

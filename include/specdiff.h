@@ -19,8 +19,9 @@
  *   - Arguments are validated on the host before anything is launched; a
  *     rejected call returns a negative SDV_E* code and launches nothing.
  *   - Work is enqueued asynchronously on `stream` (a cudaStream_t; NULL = the
- *     legacy default stream).  No call synchronises, allocates device memory
- *     or traps on the device.  A launch failure returns SDV_ECUDA;
+ *     legacy default stream).  No call allocates device memory or traps on the
+ *     device, and none synchronises except sdv_sampler_run and sdv_sampler_end,
+ *     which read the number of rounds back.  A launch failure returns SDV_ECUDA;
  *     sdv_last_cuda_error() then gives the cudaError_t.
  *   - Results are a pure function of (inputs, seed, options): reductions use a
  *     fixed order and no floating-point atomics.
@@ -340,9 +341,12 @@ int sdv_em_sample(int B, int64_t d, const float *means, const float *log_weights
  * Profiling aid (not part of the method): when enabled, sdv_verify /
  * sdv_verify_ex calls made on this host thread record CUDA events on their
  * stream into a ring of `slots` entries (one call in `every`, see
- * sdv_timing_stride; every call by default): before the fused verify kernel,
- * after it, and after the separate residual kernels used for rows longer than
- * 4096 elements.  The records are ordinary stream work, so they are captured into
+ * sdv_timing_stride; every call by default): before the first kernel of the
+ * call, after it (the fused verify kernel; with B >= 512 chains the streaming
+ * kernel of the many-chain path), and after the kernels that follow it (the
+ * many-chain finishing kernel, and the separate residual kernels used for rows
+ * longer than 4096 elements).  Calls made by sdv_sampler_run / sdv_sampler_round
+ * are not recorded.  The records are ordinary stream work, so they are captured into
  * a CUDA graph like the kernels (an event record costs a few microseconds of
  * graph time, hence the stride).  The events are created here (host objects; no
  * device memory).  slots = 0 disables timing and destroys the events.
@@ -358,10 +362,12 @@ int sdv_timing_stride(int every);
 /*
  * Waits for the events of the last `n_calls` recorded calls (1 <= n_calls <=
  * slots) and writes their summed phase times in milliseconds:
- * ms3[0] the fused verify kernel (log-ratio pass, acceptance, U-draw and, for
- * rows up to 4096 elements, the residual write), ms3[1] the long-row residual
- * kernels (0 otherwise), ms3[2] reserved (0).  SDV_EINVAL if timing is off or
- * fewer calls were recorded.
+ * ms3[0] the first kernel (the fused verify kernel: log-ratio pass, acceptance,
+ * U-draw and, for rows up to 4096 elements, the residual write; or, with B >= 512,
+ * the many-chain streaming kernel), ms3[1] the kernels after it (the many-chain
+ * finishing kernel and the long-row residual kernels; the time of the event
+ * records alone when there are none), ms3[2] reserved (0).  SDV_EINVAL if timing
+ * is off or fewer calls were recorded.
  */
 int sdv_timing_read(int n_calls, float *ms3);
 

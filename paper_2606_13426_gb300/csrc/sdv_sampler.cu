@@ -325,6 +325,9 @@ __device__ __forceinline__ RoundRow round_row(int64_t slot, int64_t slots, const
   return R;
 }
 
+// Resident CTAs per SM k_round_target_reg is built for (its register budget).
+constexpr int round_reg_blocks(int maxc) { return maxc <= 8 ? 3 : 2; }
+
 // Parallel target call of a round for rows of up to 4 kGmmThreads elements
 // (d % 4 == 0, 16-byte aligned rows): each thread owns one group of four elements
 // and holds that group of every mean in registers for the whole kernel; a CTA takes
@@ -334,9 +337,6 @@ __device__ __forceinline__ RoundRow round_row(int64_t slot, int64_t slots, const
 // resolves the next batch's rows and their schedule constants into shared memory
 // (three buffers: the batch being written, the one being finished and the next),
 // and every thread loads the next batch's states while this batch finishes.
-// Resident CTAs per SM k_round_target_reg is built for (its register budget).
-constexpr int round_reg_blocks(int maxc) { return maxc <= 8 ? 3 : 2; }
-
 template <int MAXC>
 __global__ void __launch_bounds__(kGmmThreads, round_reg_blocks(MAXC))
 k_round_target_reg(const float* __restrict__ y, const float* __restrict__ x_draft,

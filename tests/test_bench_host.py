@@ -1,0 +1,47 @@
+"""bench.py's host-side accounting, checked on the CPU: launches per call, algorithmic
+bytes of the first kernel, the shared workload name of both arms, and the lookup of a
+profile's traffic (only for the workload's full batch and a matching source hash)."""
+import os
+import re
+
+import bench
+import workloads as W
+
+
+class _Args:
+    def __init__(self, workload, mode):
+        self.workload, self.mode = workload, mode
+
+
+def test_launches_per_call():
+    assert bench.launches_per_step(256, 3072) == 1      # fused kernel (tickets reset by a memset)
+    assert bench.launches_per_step(64, 16384) == 3      # + long-row dot and write
+    assert bench.launches_per_step(1024, 3072) == 2     # k_tiles + k_finish
+    assert bench.launches_per_step(1024, 16384) == 4
+
+
+def test_algorithmic_bytes_of_the_first_kernel():
+    # pixel: window + rejected rows (read m^q, m^p) + y, all fp32
+    assert bench.fused_kernel_bytes(256, 8, 3072, "f32") == 3 * 256 * 8 * 3072 * 4 + 3 * 256 * 3072 * 4
+    # long rows and the many-chain streaming kernel move the window alone
+    assert bench.fused_kernel_bytes(64, 16, 16384, "bf16") == 3 * 64 * 16 * 16384 * 2
+    assert bench.fused_kernel_bytes(1024, 8, 3072, "f32") == 3 * 1024 * 8 * 3072 * 4
+
+
+def test_both_arms_name_the_workload_alike():
+    cfg = W.VERIFY_CONFIGS["pixel"]
+    name = bench.workload_name(_Args("pixel", "block"), cfg["B"], cfg["L"], cfg["d"], cfg["dtype"])
+    assert name == "pixel verify (B=256, L=8, d=3072 f32), block mode"
+
+
+def test_profile_traffic_lookup():
+    txt = open(os.path.join(bench.ROOT, "profiles", "k_verify_pixel.md")).read()
+    recorded = float(re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt).group(1))
+    digest = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt).group(1)
+    got = bench.profile_traffic("pixel", True)
+    assert got == (recorded if digest == bench.kernel_sources_digest() else None)
+    assert bench.profile_traffic("pixel", False) is None     # not the workload's full batch
+    assert bench.profile_traffic("tiny", True) is None       # no summary for this workload
+    # traffic, when reported, is the window plus at most the rejected rows and y
+    if got is not None:
+        assert 3 * 256 * 8 * 3072 * 4 <= got <= 1.02 * bench.fused_kernel_bytes(256, 8, 3072, "f32")

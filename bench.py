@@ -331,6 +331,25 @@ def run_sampler_rounds(args, rank, local):
                           "config": {"B": Bn, "d": d, "rounds": R}, "runs": runs}))
 
 
+def cpu_sampler_rates(n_chains, L=4, mode="block"):
+    """The oracle sampler and the oracle's plain Euler-Maruyama chain on the first
+    n_chains chains of the sampler workload (one thread): denoising steps/s of each."""
+    from oracle import sampler as OS
+    from oracle import verify as OV
+    cfg = W.SAMPLER_CONFIG
+    gm = W.make_gmm()
+    sch = OS.VPSchedule(cfg["K"], cfg["churn"], cfg["beta_min"], cfg["beta_max"], cfg["t_floor"])
+    chains = np.arange(n_chains)
+    m = OV.MODE_BLOCK if mode == "block" else OV.MODE_SAMPLE
+    t0 = time.perf_counter()
+    OS.speculative_sample(cfg["B"], cfg["d"], L, m, gm, sch, seed=100, chains=chains)
+    t_spec = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    OS.em_sample(cfg["B"], cfg["d"], gm, sch, 1, chains=chains)
+    t_em = time.perf_counter() - t0
+    return n_chains * cfg["K"] / t_spec, n_chains * cfg["K"] / t_em, t_spec, t_em
+
+
 def run_sampler(args, world, rank, local):
     """End-to-end speculative sampler on the analytic 8-component mixture (B = 1024 chains,
     d = 1024, K = 1000 VP Euler-Maruyama steps, churn 0.5, Free and Frozen drafters)
@@ -385,6 +404,14 @@ def run_sampler(args, world, rank, local):
                                "Free and Frozen drafters" % (d, Bn, K, cfg["churn"]), "best": best_key},
         "em_ms": 1e3 * t_em, "em_steps_per_s": Bn * K / t_em, "runs": runs,
     }
+    if rank == 0 and not args.skip_cpu:
+        n_cpu = 8
+        spec_rate, em_rate, t_spec, t_em_cpu = cpu_sampler_rates(n_cpu)
+        line["cpu_baseline"] = {
+            "value": spec_rate, "unit": "denoising steps/s", "cores": 1, "kind": "oracle",
+            "sample": "%d of the %d chains through oracle.sampler.speculative_sample (L=4, block, "
+                      "Free drafter; numpy fp64, one thread), %.1f s; the oracle's plain EM chain on "
+                      "the same chains: %.4g denoising steps/s (%.1f s)" % (n_cpu, Bn, t_spec, em_rate, t_em_cpu)}
     if rank == 0:
         print(json.dumps(line))
 

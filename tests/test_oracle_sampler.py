@@ -2,8 +2,11 @@
 chain and the speculative samplers (Free / Frozen drafter, sample / block verification).
 
 Independent references: quadrature of beta, finite differences of the mixture
-log-density (scipy), the closed-form law of the linear (one-component) chain, and the
-paper's remark that the Frozen drafter's first draft is always accepted.
+log-density (scipy), the closed-form law of the linear (one-component) chain, the
+paper's remark that the Frozen drafter's first draft is always accepted, and the data
+law itself: for Gaussian data the reverse chain must reach N(mu, s^2 I) at first order
+in 1/K for every churn (this pins the drift and the noise scale of the target mean
+against the forward process alone; planted misreadings of either fail it).
 """
 import math
 
@@ -126,3 +129,93 @@ def test_speculative_and_em_agree_on_the_mixture():
         y_sp = S.speculative_sample(n, 4, 5, mode, gmm, sch, seed=12)["y"]
         for u in dirs:
             assert stats.ks_2samp(y_em @ u, y_sp @ u).pvalue > 1e-3
+
+
+# ---- the reverse-SDE drift against the data law (Eq. forward-process, Eq. backward-process)
+#
+# For Gaussian data N(mu, s^2 I) the forward process has the closed-form marginals
+# q_t = N(sqrt(abar_t) mu, (abar_t s^2 + 1 - abar_t) I).  For every churn eps, the
+# reverse SDE with drift -f y + (1 + eps^2)/2 g^2 score and diffusion eps g, started
+# from q_1, has the marginals q_{1-t}; at the end of sampling that is the data law
+# itself.  The oracle's Euler-Maruyama chain must therefore reach N(mu, s^2 I) with
+# an error of first order in delta = 1/K.  With one component the oracle's target
+# mean is affine in y, so the law of Y_K is propagated exactly (mean and covariance)
+# through target_mean and VPSchedule.sigma as they stand; the only inputs that do not
+# come from the oracle's reverse-time code are q_1 (the forward closed form) and the
+# data law.  The forward-time floor (1e-4) touches only the last steps of K = 1e5 and
+# its bias is below the first-order error there.
+
+def _propagate_law(K, churn, mu, s2, target_mean=S.target_mean, sigma=None):
+    sch = S.VPSchedule(K=K, churn=churn)
+    gmm = dict(means=np.asarray(mu, np.float64)[None], log_weights=np.zeros(1), comp_var=s2)
+    d = len(mu)
+    ab1 = float(sch.alpha_bar(1.0))
+    m = math.sqrt(ab1) * np.asarray(mu, np.float64)
+    P = (ab1 * s2 + 1.0 - ab1) * np.eye(d)
+    basis = np.vstack([np.zeros(d), np.eye(d)])      # y = 0 and the unit vectors
+    for k in range(K):
+        out, _ = target_mean(basis, np.full(d + 1, k), gmm, sch)
+        c = out[0]
+        A = (out[1:] - c).T                           # m^q_k(y) = A y + c
+        sk = float(sch.sigma(k)) if sigma is None else sigma(sch, k)
+        m = A @ m + c
+        P = A @ P @ A.T + sk * sk * np.eye(d)
+    return m, P
+
+
+def _law_error(m, P, mu, s2):
+    return (np.abs(m - mu).max(), np.abs(np.diag(P) - s2).max(),
+            np.abs(P - np.diag(np.diag(P))).max())
+
+
+_MU = np.array([1.5, -2.0, 0.5])
+
+
+@pytest.mark.parametrize("s2", [0.5, 2.0])
+@pytest.mark.parametrize("churn", [0.0, 0.5, 1.5])
+def test_reverse_chain_reaches_the_data_law(s2, churn):
+    errs = []
+    for K in (1000, 10000):
+        em, ev, eo = _law_error(*_propagate_law(K, churn, _MU, s2), _MU, s2)
+        assert eo < 1e-12
+        assert max(em, ev) < 4.0 / K, (K, em, ev)
+        errs.append(max(em, ev))
+    # first order in delta: ten times more steps, ten times less error
+    assert 8.0 < errs[0] / errs[1] < 12.5, errs
+
+
+def test_reverse_chain_reaches_the_data_law_at_1e5_steps():
+    em, ev, _ = _law_error(*_propagate_law(100000, 0.5, _MU, 0.5), _MU, 0.5)
+    assert max(em, ev) < 4e-5, (em, ev)
+
+
+def _planted_flipped_f(y, k, gmm, sched):
+    """target_mean with the sign of f reversed (a planted mistake)."""
+    y = np.asarray(y, np.float64)
+    tf = sched.tfwd(k)
+    b = np.broadcast_to(sched.beta(tf), y.shape[:-1])[..., None]
+    s = S.gmm_score(y, tf, gmm["means"], gmm["log_weights"], gmm["comp_var"], sched)
+    return y + sched.delta * (-0.5 * b * y + 0.5 * (1.0 + sched.churn ** 2) * b * s), s
+
+
+def _planted_no_churn_factor(y, k, gmm, sched):
+    """target_mean without the (1 + eps^2)/2 factor on the score term (a planted mistake)."""
+    y = np.asarray(y, np.float64)
+    tf = sched.tfwd(k)
+    b = np.broadcast_to(sched.beta(tf), y.shape[:-1])[..., None]
+    s = S.gmm_score(y, tf, gmm["means"], gmm["log_weights"], gmm["comp_var"], sched)
+    return y + sched.delta * (0.5 * b * y + b * s), s
+
+
+def _planted_sigma_without_sqrt_delta(sched, k):
+    return sched.churn * math.sqrt(float(sched.beta(sched.tfwd(k))))
+
+
+@pytest.mark.parametrize("churn", [0.5, 1.5])
+def test_drift_pin_catches_planted_mistakes(churn):
+    """The pin above fails, by far, for each plausible misreading of the drift or noise."""
+    K, s2 = 10000, 0.5
+    for kw in (dict(target_mean=_planted_flipped_f), dict(target_mean=_planted_no_churn_factor),
+               dict(sigma=_planted_sigma_without_sqrt_delta)):
+        em, ev, _ = _law_error(*_propagate_law(K, churn, _MU, s2, **kw), _MU, s2)
+        assert max(em, ev) > 0.1, kw

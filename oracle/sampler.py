@@ -170,7 +170,7 @@ def speculative_sample(B, d, L, mode, gmm, sched, seed, drafter="free", chains=N
         s_bonus = sched.sigma(k + g)
         res = V.verify(x, mq, mp, np.where(sg > 0, sg, 1.0), seed_r, mode, Leff=g,
                        mu_target_bonus=mq_bonus, sigma_bonus=s_bonus,
-                       chains=None)
+                       chain_ids=chains)
         tau = res["tau"]
         # chains whose window reaches the end take no bonus step: they stop at yhat_{k+g}
         end = active & (tau == g + 1) & (k + g >= K)

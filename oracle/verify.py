@@ -231,12 +231,15 @@ def reflection_residual(Delta, Z, mq, sigma):
 # --------------------------------------------------------------------------
 def verify(x_draft, mu_target, mu_draft, sigma, seed, mode, Leff=None,
            mu_target_bonus=None, sigma_bonus=None, residual=RESIDUAL_DECOMPOSITION,
-           omega=1.0, chains=None, xtol=1e-12):
+           omega=1.0, chains=None, xtol=1e-12, chain_ids=None):
     """Run the verification step on chains ``chains`` (default: all) of a [B, L, d] window.
 
     x_draft: yhat_{k+1..k+L}; mu_target: m^q_{k..k+L-1}; mu_draft: m^p_{k..k+L-1};
     sigma: [B, L] (sigma_{k..k+L-1}).  Arrays may be any float dtype (widened to fp64).
     Leff: [B] window lengths gamma_k (default L; 0 marks an inactive chain).
+    chain_ids: the chain indices that key the random numbers of the selected rows
+    (default: ``chains`` itself); a caller that holds a subset of a larger batch in
+    compact arrays passes the subset's indices in the full batch here.
     Returns a dict of per-chain results for the selected chains, in the order given.
     """
     x_draft = np.asarray(x_draft)
@@ -246,6 +249,8 @@ def verify(x_draft, mu_target, mu_draft, sigma, seed, mode, Leff=None,
     chains = np.arange(B) if chains is None else np.asarray(chains, dtype=np.int64)
     n = len(chains)
     g = Leff[chains]
+    ids = chains if chain_ids is None else np.asarray(chain_ids, dtype=np.int64)
+    assert len(ids) == n
 
     xs = np.asarray(x_draft[chains], dtype=np.float64)
     mqs = np.asarray(np.asarray(mu_target)[chains], dtype=np.float64)
@@ -258,7 +263,7 @@ def verify(x_draft, mu_target, mu_draft, sigma, seed, mode, Leff=None,
     status = np.zeros(n, dtype=np.int64)
     bad = ~(np.isfinite(ell) & np.isfinite(dnorm)).all(axis=1)
     status[bad] |= STATUS_NONFINITE
-    eta = philox.coins(seed, chains, L)
+    eta = philox.coins(seed, ids, L)
 
     if mode == MODE_SAMPLE:
         tau = sample_verification(ell, eta, g, omega)
@@ -278,18 +283,18 @@ def verify(x_draft, mu_target, mu_draft, sigma, seed, mode, Leff=None,
     Dn = np.sqrt(np.sum(Delta * Delta, axis=-1))
     zero = resid & (Dn == 0.0)
     status[zero] |= STATUS_ZERO_DELTA
-    G = philox.normals(seed, chains, d, philox.STREAM_RESID)
+    G = philox.normals(seed, ids, d, philox.STREAM_RESID)
     y[zero] = mq_r[zero] + s_r[zero, None] * G[zero]
     dec = resid & ~zero
     if residual == RESIDUAL_REFLECTION:
         y[dec] = reflection_residual(Delta[dec], Z[dec], mq_r[dec], s_r[dec])
     elif np.any(dec):
-        w = philox.usample_uniform(seed, chains[dec])
+        w = philox.usample_uniform(seed, ids[dec])
         U[dec] = usample_bisection(Dn[dec], la_res[dec], w, xtol=xtol)
         y[dec] = decomposition_residual(Delta[dec], mq_r[dec], s_r[dec], U[dec], G[dec])
     full = (g > 0) & (tau == g + 1)
     if mu_target_bonus is not None:
-        Gb = philox.normals(seed, chains, d, philox.STREAM_BONUS)
+        Gb = philox.normals(seed, ids, d, philox.STREAM_BONUS)
         mqb = np.asarray(np.asarray(mu_target_bonus)[chains], dtype=np.float64)
         sb = np.asarray(sigma_bonus, dtype=np.float64)[chains]
         y[full] = mqb[full] + sb[full, None] * Gb[full]

@@ -219,3 +219,20 @@ def test_drift_pin_catches_planted_mistakes(churn):
                dict(sigma=_planted_sigma_without_sqrt_delta)):
         em, ev, _ = _law_error(*_propagate_law(K, churn, _MU, s2, **kw), _MU, s2)
         assert max(em, ev) > 0.1, kw
+
+
+@pytest.mark.parametrize("mode,drafter", [(V.MODE_SAMPLE, "free"), (V.MODE_BLOCK, "frozen")])
+def test_chain_subset_equals_rows_of_the_full_run(mode, drafter):
+    """Random numbers are keyed by chain index, so sampling a subset of the chains (as the
+    GPU parity tests do at full batch size) gives exactly those rows of the full run."""
+    sch = S.VPSchedule(K=25, churn=0.5)
+    gmm = _gmm(3, 5, 13)
+    full = S.speculative_sample(12, 5, 4, mode, gmm, sch, seed=14, drafter=drafter,
+                                return_trace=True)
+    sub = np.array([1, 4, 5, 11])
+    part = S.speculative_sample(12, 5, 4, mode, gmm, sch, seed=14, drafter=drafter, chains=sub,
+                                return_trace=True)
+    np.testing.assert_array_equal(part["y"], full["y"][sub])
+    np.testing.assert_array_equal(part["k"], full["k"][sub])
+    for tp, tf in zip(part["trace"], full["trace"]):
+        np.testing.assert_array_equal(tp["tau"], tf["tau"][sub])

@@ -4,8 +4,8 @@ Layout:
   csrc/       CUDA kernels and the C-ABI (libspecdiff.so, declared in include/specdiff.h)
   buildlib.py nvcc build of libspecdiff.so (in-tree, lib/)
   binding.py  ctypes binding, one Python function per C entry point, same names
-  api.py      torch-facing helpers (allocation + pointer passing only)
-  sampler.py  end-to-end speculative sampler driver over the C ABI
+  api.py      torch-facing helpers (allocation + pointer passing only), including the
+              end-to-end sampler's calls (the round loop itself runs in csrc/sdv_sampler.cu)
 
 Nothing here computes on the CPU: when the library is missing every call raises.
 """

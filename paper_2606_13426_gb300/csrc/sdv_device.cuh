@@ -334,6 +334,58 @@ static __device__ SDV_HELPER float usample_log_1mpsi(float t, const UParams& P) 
   return lA + log1mexp(lB - lA) - P.lv;
 }
 
+// log psi(a+ - t) (the residual's density at u = a+ - t), in the form whose terms do
+// not cancel: a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)) keeps every term
+// small when t is small (the deep left tail), while log alpha + log phi(u) +
+// log(1 - e^{-D t}) - log v does when u is moderate and D t is large (large |Delta|,
+// where the first form cancels terms of size D^2/2).
+__device__ __forceinline__ float usample_log_density(float t, const UParams& P) {
+  const float u = P.ap - t;
+  const float mag1 = fmaxf(fabsf(P.am * t), fmaxf(0.5f * t * t, P.D * t));
+  const float mag2 = fmaxf(0.5f * u * u, fmaxf(fabsf(P.la), fabsf(P.lv)));
+  if (mag1 <= mag2) return P.am * t - 0.5f * t * t + logexpm1(P.D * t) - P.lvn;
+  return P.la - 0.5f * u * u - kHalfLog2Pi + log1mexp(-P.D * t) - P.lv;
+}
+
+// Bracket widths (in t, i.e. in u) above which one Newton step from the bracket is not
+// accurate enough: the residual's bulk has unit scale, so a bracket of 1e-2 leaves an
+// error of ~1e-4 after one step and ~1e-8 after two.  The multisection leaves brackets
+// of about 3.5e-4 t, wider than this only for t above ~30, i.e. |Delta| of ~60 and more.
+constexpr float kUPolishWidth = 1e-2f;
+constexpr int kUPolishIters = 8;
+
+// Newton step from the end of [lo, hi] with the smaller |gap|, clamped to the bracket;
+// returns u = a+ - t directly (u_e = fl(a+ - t_e) is the point the evaluator used, so
+// the correction keeps U's rounding relative to |U| rather than to |a+|).
+__device__ __forceinline__ float usample_newton(const UParams& P, bool upper, float target, float lo,
+                                                float glo, float hi, float ghi) {
+  const bool from_lo = isfinite(glo) && (-glo < ghi);
+  const float te = from_lo ? lo : hi, ge = from_lo ? glo : ghi;
+  const float lpsi = usample_log_density(te, P);
+  const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
+  const float dg = expf(lpsi - lden);
+  const float ue = P.ap - te;
+  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
+  step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
+  return ue + step;
+}
+
+// While the bracket is wider than kUPolishWidth: evaluate the gap at the Newton point
+// (the bracket's midpoint if that point is not strictly inside) and keep the half that
+// holds the root (safeguarded Newton).  Every thread passes and gets the same values.
+template <typename Gap>
+__device__ __forceinline__ void usample_polish(const UParams& P, bool upper, float target, const Gap& gap,
+                                               float& lo, float& glo, float& hi, float& ghi) {
+#pragma unroll 1
+  for (int it = 0; it < kUPolishIters && hi - lo > kUPolishWidth; ++it) {
+    float t = P.ap - usample_newton(P, upper, target, lo, glo, hi, ghi);
+    if (!(t > lo && t < hi)) t = 0.5f * (lo + hi);
+    const float gt = gap(t);
+    if (!(gt == gt)) break;
+    if (gt >= 0.0f) { hi = t; ghi = gt; } else { lo = t; glo = gt; }
+  }
+}
+
 // Shared scratch of usample_block.
 struct USampleScratch {
   int first[32];
@@ -351,9 +403,11 @@ struct USampleScratch {
 //     bracket, eight steps per octave, all at once), s0 = 1/max(1, |a-|) the
 //     scale of the residual's spread;
 //  2. one round of NT-way multisection;
-//  3. one Newton step from the bracket end with the smaller |g|, clamped to the
-//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form,
-//     log psi(a+ - t) = a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)).
+//  3. while the bracket is wider than kUPolishWidth (large |Delta| only), safeguarded
+//     Newton steps with the gap evaluated at each new point;
+//  4. one Newton step from the bracket end with the smaller |g|, clamped to the
+//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form
+//     (usample_log_density).
 template <int NT>
 __device__ __forceinline__ float usample_block(const UParams& P, uint32_t wbits, uint32_t* status,
                                                USampleScratch* sm) {
@@ -404,18 +458,8 @@ __device__ __forceinline__ float usample_block(const UParams& P, uint32_t wbits,
     ghi = sm->g[1];
     __syncthreads();
   }
-  // Newton step from the closer end
-  const bool from_lo = isfinite(glo) && (-glo < ghi);
-  const float te = from_lo ? lo : hi, ge = from_lo ? glo : ghi;
-  const float lpsi = P.am * te - 0.5f * te * te + logexpm1(P.D * te) - P.lvn;
-  const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
-  const float dg = expf(lpsi - lden);
-  // Return u directly: u_e = fl(a+ - t_e) is the point the evaluator used, so adding
-  // the Newton correction keeps U's rounding relative to |U| rather than to |a+|.
-  const float ue = P.ap - te;
-  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
-  step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
-  return ue + step;
+  usample_polish(P, upper, target, gap, lo, glo, hi, ghi);
+  return usample_newton(P, upper, target, lo, glo, hi, ghi);
 }
 
 // U = Psi_alpha^{-1}(w), w = (wbits + 1/2) 2^-32, by one converged warp: every lane
@@ -426,9 +470,11 @@ __device__ __forceinline__ float usample_block(const UParams& P, uint32_t wbits,
 //  1. bracket: the 32 candidates t_k = s0 2^(k - 8) (the paper's doubling of the
 //     bracket, all steps at once), s0 = 1/max(1, |a-|) the residual's scale;
 //  2. kURounds rounds of 32-way multisection (each shrinks the bracket 32-fold);
-//  3. one Newton step from the bracket end with the smaller |g|, clamped to the
-//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form,
-//     log psi(a+ - t) = a- t - t^2/2 + log expm1(D t) - (log v - log phi(a-)).
+//  3. while the bracket is wider than kUPolishWidth (large |Delta| only), safeguarded
+//     Newton steps with the gap evaluated at each new point;
+//  4. one Newton step from the bracket end with the smaller |g|, clamped to the
+//     bracket.  g' = psi / Psi (or psi / (1 - Psi)) with the density in closed form
+//     (usample_log_density).
 constexpr int kURounds = 3;
 
 __device__ __forceinline__ float usample_warp(const UParams& P, uint32_t wbits, uint32_t* status) {
@@ -468,18 +514,8 @@ __device__ __forceinline__ float usample_warp(const UParams& P, uint32_t wbits, 
     hi = nt;
     ghi = ng;
   }
-  // Newton step from the closer end
-  const bool from_lo = isfinite(glo) && (-glo < ghi);
-  const float te = from_lo ? lo : hi, ge = from_lo ? glo : ghi;
-  const float lpsi = P.am * te - 0.5f * te * te + logexpm1(P.D * te) - P.lvn;
-  const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
-  const float dg = expf(lpsi - lden);
-  // Return u directly: u_e = fl(a+ - t_e) is the point the evaluator used, so adding
-  // the Newton correction keeps U's rounding relative to |U| rather than to |a+|.
-  const float ue = P.ap - te;
-  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
-  step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
-  return ue + step;
+  usample_polish(P, upper, target, gap, lo, glo, hi, ghi);
+  return usample_newton(P, upper, target, lo, glo, hi, ghi);
 }
 
 // ---------------------------------------------------------------- tickets

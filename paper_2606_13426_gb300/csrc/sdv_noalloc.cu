@@ -12,11 +12,9 @@
 // The scratch is a file-scope __device__ array of SDV_NOALLOC_SCRATCH_BYTES.  Every
 // GPU on which this library is loaded holds it until the process exits.  Host code
 // cannot use the array's name as a device address (it is a host-side stand-in), so
-// the device address is fetched with cudaGetSymbolAddress, once per device, with
-// that device current, and passed to the kernels as their workspace.
+// the device address is fetched with cudaGetSymbolAddress, on every call with the
+// caller's device current, and passed to the kernels as their workspace.
 #include <cuda_runtime.h>
-
-#include <mutex>
 
 #include "sdv_host.h"
 
@@ -24,25 +22,15 @@ namespace {
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[SDV_NOALLOC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_noalloc_mutex;
-void* g_noalloc_ptr[kMaxDevices] = {};
-
-// Device address of the scratch on the current device (set-up on first use).
-int noalloc_scratch(void** out) {
+// Device address of the scratch on the current device.  It is looked up on every call
+// (a host-side lookup that allocates nothing): a cached address would go stale when
+// the device's primary context is torn down (cudaDeviceReset) and the module is
+// loaded again at another address.
+cudaError_t noalloc_scratch(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return (int)e;
-  if (dev < 0 || dev >= kMaxDevices) return (int)cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-  if (g_noalloc_ptr[dev] == nullptr) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return (int)e;
-    g_noalloc_ptr[dev] = p;
-  }
-  *out = g_noalloc_ptr[dev];
-  return 0;
+  if (e != cudaSuccess) return e;
+  return cudaGetSymbolAddress(out, g_noalloc_scratch);
 }
 
 }  // namespace
@@ -57,9 +45,10 @@ extern "C" int sdv_verify_noalloc(const void* x_draft, const void* mu_target, co
   if (need == 0) return SDV_EINVAL;
   if (need > (size_t)SDV_NOALLOC_SCRATCH_BYTES) return SDV_ENOWORKSPACE;
   void* scratch = nullptr;
-  const int err = noalloc_scratch(&scratch);
-  if (err != 0) {
-    cudaGetLastError();  // reset the runtime's last-error slot so a later launch check does not report it
+  if (noalloc_scratch(&scratch) != cudaSuccess) {
+    // record the failure for sdv_last_cuda_error() and clear the runtime's last-error
+    // slot, so that a later launch check does not report it again
+    sdv::set_last_cuda_error((int)cudaGetLastError());
     return SDV_ECUDA;
   }
   // The tickets that must start at zero are cleared by the call itself (a memset on

@@ -84,6 +84,41 @@ def test_usample_degenerate_inputs(api):
     assert torch.isnan(U).all()
 
 
+def test_usample_range_of_the_bracket(api):
+    """The bracket's candidates t = a+ - U reach s0 2^(255/8 - 8) with s0 = 1/max(1, |a-|)
+    (the warp version s0 2^23), which covers the residual whenever |Delta| is below about
+    5800 (at |Delta| = D and alpha = 1 the residual is close to N(0, 1) while a+ = D/2).
+    Inside that range U matches the oracle (up to the rounding of a+ itself, from which U
+    is formed in fp32); far outside it the kernel reports SDV_STATUS_USAMPLE_RANGE."""
+    wbits = [1, 12345, 2 ** 31 - 1, 2 ** 31, 3 * 2 ** 30, 2 ** 32 - 2]
+    D_in = [64.0, 512.0, 3000.0]
+    la_in = [0.0, -5.0]
+    D, la, wb = [], [], []
+    for Dv in D_in:
+        for lav in la_in:
+            for w in wbits:
+                D.append(Dv); la.append(lav); wb.append(w)
+    n_in = len(D)
+    for Dv in (2.0e4, 1.0e5):
+        for w in wbits:
+            D.append(Dv); la.append(0.0); wb.append(w)
+    D = np.array(D, np.float32)
+    la = np.array(la, np.float32)
+    wb = np.array(wb, np.uint64).astype(np.uint32)
+    U, st = api.usample(torch.from_numpy(D).cuda(), torch.from_numpy(la).cuda(),
+                        torch.from_numpy(wb.view(np.int32)).cuda())
+    U = U.cpu().numpy().astype(np.float64)
+    st = st.cpu().numpy()
+    assert np.all(st[:n_in] == 0)
+    Uo = OV.usample_bisection(D[:n_in].astype(np.float64), la[:n_in].astype(np.float64),
+                              OP.uniform_of(wb[:n_in]))
+    ap = la[:n_in] / D[:n_in] + 0.5 * D[:n_in]
+    tol = 5e-6 + 3e-7 * np.abs(Uo) + 2.0 ** -23 * np.abs(ap)
+    assert np.all(np.abs(U[:n_in] - Uo) <= tol), np.max(np.abs(U[:n_in] - Uo) / tol)
+    assert np.all(st[n_in:] & 4), st[n_in:]          # SDV_STATUS_USAMPLE_RANGE
+    assert np.all(np.isfinite(U[n_in:]))
+
+
 # ------------------------------------------------------------------ a2: log ratios
 @pytest.mark.parametrize("kind,B,L,d", [("tiny", 4, 4, 16), ("pixel", 32, 8, 3072),
                                         ("latent", 8, 16, 16384), ("pixel", 5, 3, 4099),

@@ -1,19 +1,25 @@
 """Benchmark of the speculative-diffusion verification step on GB300.
 
-One step = one sdv_verify call (one fused kernel: log-ratio pass, acceptance
-scan, residual U-draw, residual write) on one batch of the pixel-scale workload (B=256 chains,
-L=8 draft steps, d=3x32x32 fp32, block verification) with inputs resident in
-HBM.  Eight input sets (8 x 75.5 MB, well above the 129 MB L2) rotate between
-steps, so every step reads its inputs from HBM.  Steps are captured into CUDA
-graphs and replayed.
+One step = one verification call (sdv_verify_pipelined: one fused kernel -- log-ratio
+pass, acceptance rule, residual U-draw, residual write) on one batch of the
+pixel-scale workload (B=256 chains, L=8 draft steps, d=3x32x32 fp32, block
+verification) with inputs resident in HBM.  Eight input sets (8 x 75.5 MB, well
+above the 129 MB L2) rotate between steps, so every step reads its inputs from HBM.
+Steps are independent batches of chains: consecutive calls may overlap on the GPU (a
+call streams its window while the previous call's last chains finish).  Steps are
+captured into CUDA graphs and replayed.
 
 Prints ONE JSON line (rank 0):
-  value      verified draft-steps/s (B*L per step), whole job
-  roofline   the fused verify kernel (dominant kernel): algorithmic bytes / its mean
-             duration from CUDA events inside the timed region, vs measured HBM peak
-  e2e        the same metric through the public API from pinned host buffers
-             (host->device copy of the window, device->host copy of results)
-  cpu_baseline  the CPU oracle on a bounded sample of the same workload
+  value        verified draft-steps/s (B*L per step), whole job
+  roofline     full-call algorithmic bytes per call / the per-call period of 200
+               back-to-back calls in one graph (events at its two ends only), vs the
+               measured HBM copy peak
+  steady_state the per-call period over >= 1 s of replays of the timed graph
+  workloads    the same figures for the latent (bf16) and high-resolution workloads,
+               and the end-to-end sampler's wall-clock
+  e2e          the same metric through the public API from pinned host memory
+               (api.HostStream: window copied in, results copied out, every step)
+  cpu_baseline the CPU oracle on a bounded sample of the same workload
 
 --impl reference times the CPU oracle alone (the reference arm of this build).
 """
@@ -37,14 +43,13 @@ import workloads as W  # noqa: E402
 METRIC = "verified draft-steps/s and HBM GB/s vs ~8 TB/s; mean accepted steps/target call"
 UNIT = "draft-steps/s"
 N_SETS = 8
-TIMING_STRIDE = 16
 
 
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20000)
-    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="pixel", choices=["pixel", "latent", "highres", "sampler"])
     p.add_argument("--sampler-L", default="4,8,16",
@@ -56,7 +61,10 @@ def parse():
     p.add_argument("--mode", default="block", choices=["block", "sample"])
     p.add_argument("--batch", type=int, default=0,
                    help="chains per call (0: the workload's B); smaller batches serve ncu captures")
-    p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--no-pipeline", action="store_true",
+                   help="time sdv_verify_ex calls instead of sdv_verify_pipelined")
+    p.add_argument("--headline-only", action="store_true",
+                   help="skip the latent / high-resolution / sampler sub-results")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--skip-cpu", action="store_true")
     return p.parse_args()
@@ -141,14 +149,9 @@ class ClockSampler:
 
 
 # Rows of more than this many groups of four elements get their residual from two
-# extra kernels (the library's kFusedMaxGroups).
-FUSED_MAX_GROUPS = 1024
-
-
-def long_rows(d):
-    """Rows longer than 4 FUSED_MAX_GROUPS elements get their residual from two extra kernels."""
-    return (d + 3) // 4 > FUSED_MAX_GROUPS
-
+# extra kernels (the library's kFusedMaxGroups; kFinishMaxGroups on the many-chain path).
+FUSED_MAX_GROUPS = 4096
+FINISH_MAX_GROUPS = 1024
 
 # From this many chains on, the library streams the tiles with k_tiles and finishes
 # every chain with one warp of k_finish (the library's kManyChainMin).
@@ -159,20 +162,23 @@ def many_chains(B):
     return B >= MANY_CHAIN_MIN
 
 
+def long_rows(d, B=0):
+    """Rows whose residual two extra kernels write (longer than the fused kernel's, or on
+    the many-chain path k_finish's, noise cache)."""
+    return (d + 3) // 4 > (FINISH_MAX_GROUPS if many_chains(B) else FUSED_MAX_GROUPS)
+
+
 def launches_per_step(B, d):
-    """Kernels one sdv_verify call launches: the fused verify kernel (or k_tiles and
-    k_finish for many chains), plus the residual dot / write kernels for long rows
-    (the ticket reset of the fused kernel is a memset)."""
-    return (2 if many_chains(B) else 1) + (2 if long_rows(d) else 0)
+    """Kernels one verification call launches: the fused verify kernel (or k_tiles and
+    k_finish for many chains), plus the residual dot / write kernels for long rows."""
+    return (2 if many_chains(B) else 1) + (2 if long_rows(d, B) else 0)
 
 
-def fused_kernel_bytes(B, L, d, dtype):
-    """Algorithmic bytes of the first kernel of a call: x, m^q, m^p read once, and, when
-    the fused kernel also writes the residual, the rejected row's m^q and m^p (upper
-    bound: every chain) re-read plus y written."""
+def call_bytes(B, L, d, dtype):
+    """Algorithmic bytes of one call: x, m^q, m^p read once, and the residual pass: the
+    rejected row's m^q and m^p re-read plus y written (upper bound: every chain)."""
     s = W.bytes_per_element(dtype)
-    main = 3 * B * L * d * s
-    return main if (long_rows(d) or many_chains(B)) else main + 3 * B * d * s
+    return 3 * B * L * d * s + 3 * B * d * s
 
 
 def input_seed(base, i, rank):
@@ -416,6 +422,197 @@ def run_sampler(args, world, rank, local):
         print(json.dumps(line))
 
 
+def _graph_of_calls(stream, n, call):
+    """A CUDA graph of n calls call(0..n-1) captured on `stream`."""
+    import torch
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n):
+            call(i)
+    return g
+
+
+def _replay_ms(stream, graphs, reps=1):
+    """Device time of replaying `graphs` (in order, `reps` times) between two events."""
+    import torch
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(reps):
+            for g in graphs:
+                g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clocks=None, pipelined=True):
+    """Timed verification calls on workload `name`: the timed region (steps calls in CUDA
+    graph replays, events at its ends), the per-call period of 200 back-to-back calls
+    (the roofline's duration), the steady-state period over >= 1 s of replays, and mean
+    tau per target call in both modes.  Returns a dict; the input sets stay on the device
+    only while it runs."""
+    import torch
+    cfg = W.VERIFY_CONFIGS[name]
+    L, d, dt_name = cfg["L"], cfg["d"], cfg["dtype"]
+    tdt = torch.bfloat16 if dt_name == "bf16" else torch.float32
+    set_bytes = W.main_pass_bytes(Bn, L, d, dt_name)
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 129 * 2 ** 20)
+    n_sets = max(1, min(N_SETS, math.ceil(4 * l2 / set_bytes))) if set_bytes < 4 * l2 else 1
+
+    def to_dev(inp, key):
+        if dt_name == "bf16":
+            return torch.from_numpy(inp[key + "_bits"].view(np.int16)).to(dev).view(torch.bfloat16)
+        return torch.from_numpy(inp[key]).to(dev)
+
+    sets, host0 = [], None
+    for i in range(n_sets):
+        inp = W.make_verify_inputs(name, B=Bn, seed=input_seed(cfg["seed"], i, rank))
+        sets.append(dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"),
+                         mp=to_dev(inp, "mu_draft"), sigma=torch.from_numpy(inp["sigma"]).to(dev)))
+        if i == 0:
+            host0 = inp
+    outs = dict(accepted_len=torch.empty(Bn, dtype=torch.int32, device=dev),
+                y=torch.empty(Bn, d, dtype=tdt, device=dev),
+                status=torch.empty(Bn, dtype=torch.int32, device=dev))
+    ws = torch.zeros(max(api.workspace_bytes(Bn, L, d, tdt), 256), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i, m=mode):
+        st = sets[i % n_sets]
+        api.verify(st["x"], st["mq"], st["mp"], st["sigma"], seed=i, mode=m, with_ratios=False,
+                   workspace=ws, out=outs, pipelined=pipelined)
+
+    with torch.cuda.stream(stream):
+        for i in range(max(warmup, 1)):
+            step(i)
+    torch.cuda.synchronize()
+    g_steps = min(steps, 256)
+    reps, rem = divmod(steps, g_steps)
+    g_main = _graph_of_calls(stream, g_steps, step)
+    graphs = [g_main] * reps
+    if rem:
+        graphs.append(_graph_of_calls(stream, rem, step))
+    _replay_ms(stream, graphs[:1])                            # graph warm-up
+
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    ms_total = _replay_ms(stream, graphs)
+    clk = clocks.stop() if clocks else None
+    ms_total = max_over_ranks(ms_total, pg, dev)
+    if pg:
+        pg.barrier()
+    ms_step = ms_total / steps
+
+    # the roofline's duration: 200 back-to-back calls in one graph, events at its ends only
+    g200 = _graph_of_calls(stream, 200, step)
+    _replay_ms(stream, [g200])
+    ms_call = min(_replay_ms(stream, [g200]) for _ in range(3)) / 200
+    # steady state: replays of the 200-call graph for >= 1 s
+    reps_ss = max(1, int(math.ceil(1000.0 / max(ms_call * 200, 1e-3))))
+    ms_ss = _replay_ms(stream, [g200], reps=reps_ss) / (200 * reps_ss)
+
+    taus = {}
+    for m in ("block", "sample"):
+        acc = []
+        for i, st in enumerate(sets):
+            r = api.verify(st["x"], st["mq"], st["mp"], st["sigma"], seed=10_000 + i, mode=m,
+                           with_ratios=False, workspace=ws)
+            acc.append(r["accepted_len"].cpu().numpy())
+        taus[m] = float(np.concatenate(acc).mean() + 1.0)
+    del sets, g_main, graphs, g200
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+    hbm_peak, peak_kind = peaks()
+    nbytes = call_bytes(Bn, L, d, dt_name)
+    achieved = nbytes / (ms_call * 1e-3) / 1e9
+    return dict(
+        name=name, B=Bn, L=L, d=d, dtype=dt_name, n_sets=n_sets, set_bytes=set_bytes, l2=l2,
+        ms_step=ms_step, ms_call=ms_call, ms_steady=ms_ss, steady_calls=200 * reps_ss,
+        value_per_rank=Bn * L / (ms_step * 1e-3), taus=taus, clocks=clk, host0=host0,
+        roofline={"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                  "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                  "kernel": ("k_verify (fused: log-ratio pass, acceptance, U-draw, residual write)"
+                             if launches_per_step(Bn, d) == 1 else
+                             "whole call (%d kernels: %s)" % (launches_per_step(Bn, d),
+                                                             "k_tiles, k_finish" if many_chains(Bn)
+                                                             else "k_verify, k_resid_dot, k_resid_write")),
+                  "duration": "per-call period of 200 back-to-back calls in one CUDA graph "
+                              "(events at its two ends only)",
+                  "duration_us": 1e3 * ms_call, "algorithmic_bytes": nbytes,
+                  "traffic": profile_traffic(name, Bn == cfg["B"])})
+
+
+def measure_e2e(api, host0, Bn, L, d, dt_name, mode, dev, n_steps):
+    """The metric through the public API from pinned host memory: api.HostStream copies
+    each step's window in (one [3, B, L, d] copy) while the previous step verifies, and
+    copies its accepted lengths and states back; timed on the host clock."""
+    import torch
+    tdt = torch.bfloat16 if dt_name == "bf16" else torch.float32
+    win = torch.empty(3, Bn, L, d, dtype=tdt, pin_memory=True)
+    for k, key in enumerate(("x_draft", "mu_target", "mu_draft")):
+        if dt_name == "bf16":
+            win[k].view(torch.int16).copy_(torch.from_numpy(host0[key + "_bits"].view(np.int16)))
+        else:
+            win[k].copy_(torch.from_numpy(host0[key]))
+    sig = torch.from_numpy(host0["sigma"]).pin_memory()
+    hs = api.HostStream(Bn, L, d, tdt, tuple(sig.shape), depth=2, device=dev)
+    for i in range(4):
+        hs.result(hs.submit(win, sig, i, mode))
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    prev = None
+    for i in range(n_steps):
+        cur = hs.submit(win, sig, i, mode)
+        if prev is not None:
+            hs.result(prev)
+        prev = cur
+    hs.result(prev)
+    e2e_s = (time.perf_counter() - t0) / n_steps
+    h2d = win.numel() * win.element_size() + sig.numel() * 4
+    d2h = Bn * 4 + Bn * d * win.element_size()
+    return e2e_s, h2d, d2h
+
+
+def sampler_summary(api, dev):
+    """Wall-clock of the end-to-end sampler (L = 8, block, Free drafter; best of three)
+    against the plain Euler-Maruyama chain, on the sampler workload."""
+    import torch
+    cfg = W.SAMPLER_CONFIG
+    gm = W.make_gmm()
+    tgt = api.GmmTarget(torch.from_numpy(gm["means"]), torch.from_numpy(gm["log_weights"]),
+                        gm["comp_var"], cfg["K"], cfg["churn"], device=dev)
+    Bn, d, K, L = cfg["B"], cfg["d"], cfg["K"], 8
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        out = fn()
+        torch.cuda.synchronize()
+        return out, time.perf_counter() - t0
+
+    timed(lambda: api.em_sample(Bn, tgt, 1))
+    t_em = min(timed(lambda: api.em_sample(Bn, tgt, 2 + i))[1] for i in range(3))
+    ws = torch.empty(api.B.sdv_sampler_workspace_bytes(Bn, L, d), dtype=torch.uint8, device=dev)
+    timed(lambda: api.sampler_run(Bn, L, tgt, 7, "block", "free", workspace=ws))
+    best = min((timed(lambda: api.sampler_run(Bn, L, tgt, 100 + i, "block", "free", workspace=ws))
+                for i in range(3)), key=lambda rt: rt[1])
+    r, t = best
+    cr = r["chain_rounds"].cpu().numpy().astype(np.float64)
+    ts = r["tau_sum"].cpu().numpy().astype(np.float64)
+    return {"workload": "analytic 8-component GMM, d=%d, B=%d, K=%d, L=%d, block, Free drafter"
+                        % (d, Bn, K, L),
+            "ms": 1e3 * t, "rounds": r["rounds"], "mean_tau": float(ts.sum() / cr.sum()),
+            "denoising_steps_per_s": Bn * K / t, "em_ms": 1e3 * t_em}
+
+
 def main():
     args = parse()
     world, rank, local = dist_setup()
@@ -432,7 +629,7 @@ def main():
     import torch
     import __graft_entry__ as G
     G.build()
-    from paper_2606_13426_gb300 import api, binding
+    from paper_2606_13426_gb300 import api
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
@@ -443,174 +640,67 @@ def main():
         pg = dist
 
     cfg = W.VERIFY_CONFIGS[args.workload]
-    Bn, L, d, dt_name = cfg["B"], cfg["L"], cfg["d"], cfg["dtype"]
-    if args.batch > 0:
-        Bn = args.batch
-    tdt = torch.bfloat16 if dt_name == "bf16" else torch.float32
-    set_bytes = W.main_pass_bytes(Bn, L, d, dt_name)
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size if hasattr(
-        torch.cuda.get_device_properties(dev), "L2_cache_size") else 129 * 2 ** 20
-    n_sets = max(1, min(N_SETS, math.ceil(4 * l2 / set_bytes))) if set_bytes < 4 * l2 else 1
-
-    def to_dev(inp, name):
-        if dt_name == "bf16":
-            return torch.from_numpy(inp[name + "_bits"].view(np.int16)).to(dev).view(torch.bfloat16)
-        return torch.from_numpy(inp[name]).to(dev)
-
-    sets = []
-    host0 = None
-    for i in range(n_sets):
-        inp = W.make_verify_inputs(args.workload, B=Bn, seed=input_seed(cfg["seed"], i, rank))
-        sets.append(dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"),
-                         mp=to_dev(inp, "mu_draft"), sigma=torch.from_numpy(inp["sigma"]).to(dev)))
-        if i == 0:
-            host0 = inp
-    outs = dict(accepted_len=torch.empty(Bn, dtype=torch.int32, device=dev),
-                y=torch.empty(Bn, d, dtype=tdt, device=dev),
-                status=torch.empty(Bn, dtype=torch.int32, device=dev))
-    ws = api.make_workspace(Bn, L, d, tdt, dev)
-    stream = torch.cuda.Stream(device=dev)
-
-    def step(i):
-        s = sets[i % n_sets]
-        api.verify(s["x"], s["mq"], s["mp"], s["sigma"], seed=i, mode=args.mode,
-                   with_ratios=False, workspace=ws, out=outs)
-
-    G_STEPS = min(args.steps, 256)
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            step(i)
-    torch.cuda.synchronize()
-    # kernel durations from events on one call in TIMING_STRIDE inside the timed
-    # region (an event record costs a few microseconds of graph time)
-    binding.sdv_timing_enable(G_STEPS)
-    binding.sdv_timing_stride(TIMING_STRIDE)
-
-    graphs = []
-    use_graph = not args.no_graph
-    if use_graph:
-        try:
-            reps, rem = divmod(args.steps, G_STEPS)
-            g_main = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g_main, stream=stream):
-                for i in range(G_STEPS):
-                    step(i)
-            graphs = [g_main] * reps
-            if rem:
-                g_rem = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g_rem, stream=stream):
-                    for i in range(rem):
-                        step(i)
-                graphs.append(g_rem)
-            for g in graphs[:1]:
-                g.replay()
-            torch.cuda.synchronize()
-        except Exception as e:  # capture unsupported: time eager launches instead
-            sys.stderr.write("graph capture failed (%s); timing eager launches\n" % e)
-            use_graph = False
-            torch.cuda.synchronize()
-
+    Bn = args.batch if args.batch > 0 else cfg["B"]
+    L, d, dt_name = cfg["L"], cfg["d"], cfg["dtype"]
+    pipelined = not args.no_pipeline
     clocks = ClockSampler(local)
-    if pg:
-        pg.barrier()
-    torch.cuda.synchronize()
-    clocks.start()
-    time.sleep(0.3)
-    ev0 = torch.cuda.Event(enable_timing=True)
-    ev1 = torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        ev0.record(stream)
-        if use_graph:
-            for g in graphs:
-                g.replay()
-        else:
-            for i in range(args.steps):
-                step(i)
-        ev1.record(stream)
-    torch.cuda.synchronize()
-    ms_total = ev0.elapsed_time(ev1)
-    clk = clocks.stop()
-    last_len = (args.steps % G_STEPS or G_STEPS) if use_graph else min(args.steps, G_STEPS)
-    n_timed = max(1, -(-last_len // TIMING_STRIDE))
-    kv_ms, kr_ms, _ = (v / n_timed for v in binding.sdv_timing_read(n_timed))
-    binding.sdv_timing_enable(0)
-    ms_total = max_over_ranks(ms_total, pg, dev)
-    if pg:
-        pg.barrier()
-    ms_step = ms_total / args.steps
-    value = whole_job_rate(world, Bn * L, ms_step * 1e-3)
+    head = measure_verify(api, args.workload, Bn, args.mode, args.steps, args.warmup, dev, rank, pg,
+                          clocks, pipelined)
+    value = whole_job_rate(world, Bn * L, head["ms_step"] * 1e-3)
 
-    # mean tau per target call, block and sample, over the input sets
-    taus = {}
-    for mode in ("block", "sample"):
-        acc = []
-        for i, s in enumerate(sets):
-            r = api.verify(s["x"], s["mq"], s["mp"], s["sigma"], seed=10_000 + i, mode=mode,
-                           with_ratios=False, workspace=ws)
-            acc.append(r["accepted_len"].cpu().numpy())
-        taus[mode] = float(np.concatenate(acc).mean() + 1.0)
+    subs = {}
+    if not args.headline_only:
+        for name in ("latent", "highres"):
+            if name == args.workload:
+                continue
+            c = W.VERIFY_CONFIGS[name]
+            r = measure_verify(api, name, c["B"], args.mode, args.steps, args.warmup, dev, rank, pg,
+                               None, pipelined)
+            subs[name] = {
+                "workload": workload_name(argparse.Namespace(workload=name, mode=args.mode), c["B"], c["L"],
+                                          c["d"], c["dtype"]),
+                "value": whole_job_rate(world, c["B"] * c["L"], r["ms_step"] * 1e-3), "unit": UNIT,
+                "ms_per_step": r["ms_step"], "steady_state_ms_per_step": r["ms_steady"],
+                "hbm_gbs_step": r["roofline"]["algorithmic_bytes"] / (r["ms_step"] * 1e-3) / 1e9,
+                "roofline": r["roofline"], "mean_tau_block": r["taus"]["block"],
+                "mean_tau_sample": r["taus"]["sample"],
+                "gpu_launches": launches_per_step(c["B"], c["d"]) * args.steps}
+        subs["sampler"] = sampler_summary(api, dev)
 
-    # end to end: pinned host window in, accepted lengths and states out
-    sig_shape = tuple(host0["sigma"].shape)
-    hx = torch.empty(Bn, L, d, dtype=tdt, pin_memory=True)
-    hq = torch.empty_like(hx, pin_memory=True)
-    hp = torch.empty_like(hx, pin_memory=True)
-    if dt_name == "bf16":
-        for h, n in ((hx, "x_draft"), (hq, "mu_target"), (hp, "mu_draft")):
-            h.view(torch.int16).copy_(torch.from_numpy(host0[n + "_bits"].view(np.int16)))
-    else:
-        hx.copy_(torch.from_numpy(host0["x_draft"]))
-        hq.copy_(torch.from_numpy(host0["mu_target"]))
-        hp.copy_(torch.from_numpy(host0["mu_draft"]))
-    hs = torch.from_numpy(host0["sigma"]).pin_memory()
-    dbufs = api.make_device_buffers(Bn, L, d, tdt, sig_shape, device=dev)
-    e2e_steps = max(20, min(400, args.steps // 50))
-    with torch.cuda.stream(stream):
-        for i in range(3):
-            api.verify_host(hx, hq, hp, hs, i, args.mode, dev_bufs=dbufs)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        for i in range(e2e_steps):
-            api.verify_host(hx, hq, hp, hs, i, args.mode, dev_bufs=dbufs)
-        e2e_s = (time.perf_counter() - t0) / e2e_steps
-    h2d = 3 * hx.numel() * hx.element_size() + hs.numel() * 4
-    d2h = Bn * 4 + Bn * d * hx.element_size()
+    e2e_steps = max(20, min(400, args.steps))
+    e2e_s, h2d, d2h = measure_e2e(api, head["host0"], Bn, L, d, dt_name, args.mode, dev, e2e_steps)
 
-    hbm_peak, peak_kind = peaks()
-    kv_bytes = fused_kernel_bytes(Bn, L, d, dt_name)
-    achieved = kv_bytes / (kv_ms * 1e-3) / 1e9
+    nbytes = head["roofline"]["algorithmic_bytes"]
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": head["ms_step"], "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32" if dt_name == "f32" else "bf16",
         "data": "synthetic",
         "config": {"workload": workload_name(args, Bn, L, d, dt_name),
                    "global_batch": world * Bn, "window": L, "dim": d,
                    "parallelism": "replicas" if world > 1 else "single-gpu",
                    "l2": "%d rotating input sets, %.0f MB > L2 %.0f MB" % (
-                       n_sets, n_sets * set_bytes / 1e6, l2 / 1e6) if n_sets > 1 else
-                   "one input set of %.0f MB > L2" % (set_bytes / 1e6),
-                   "cuda_graph": use_graph},
-        "hbm_gbs_step": (set_bytes / (ms_step * 1e-3)) / 1e9,
-        "mean_tau_block": taus["block"], "mean_tau_sample": taus["sample"],
-        "phase_us": ({"tiles_kernel": 1e3 * kv_ms, "finish_and_residual": 1e3 * kr_ms}
-                     if many_chains(Bn) else
-                     {"verify_kernel": 1e3 * kv_ms,
-                      "long_row_residual": 1e3 * kr_ms if long_rows(d) else None}),
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "peak_kind": peak_kind,
-                     "kernel": "k_tiles (log-ratio pass of the many-chain path)" if many_chains(Bn)
-                               else "k_verify (fused: log-ratio pass, acceptance, U-draw%s)"
-                               % ("" if long_rows(d) else ", residual write"),
-                     "algorithmic_bytes": kv_bytes,
-                     "traffic": profile_traffic(args.workload, Bn == W.VERIFY_CONFIGS[args.workload]["B"])},
+                       head["n_sets"], head["n_sets"] * head["set_bytes"] / 1e6, head["l2"] / 1e6)
+                   if head["n_sets"] > 1 else "one input set of %.0f MB > L2" % (head["set_bytes"] / 1e6),
+                   "cuda_graph": True,
+                   "calls": "sdv_verify_pipelined (consecutive independent calls may overlap)"
+                            if pipelined else "sdv_verify_ex"},
+        "hbm_gbs_step": nbytes / (head["ms_step"] * 1e-3) / 1e9,
+        "steady_state": {"ms_per_step": head["ms_steady"], "calls": head["steady_calls"],
+                         "value": whole_job_rate(world, Bn * L, head["ms_steady"] * 1e-3),
+                         "hbm_gbs": nbytes / (head["ms_steady"] * 1e-3) / 1e9},
+        "mean_tau_block": head["taus"]["block"], "mean_tau_sample": head["taus"]["sample"],
+        "roofline": head["roofline"],
         "e2e": {"value": world * Bn * L / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+                "d2h_bytes_per_step": d2h,
+                "api": "api.HostStream (pinned [3,B,L,d] window in, accepted_len and y out, "
+                       "copy of step i+1 overlapping step i)"},
         "gpu_launches": launches_per_step(Bn, d) * args.steps,
-        "clocks": clk,
+        "clocks": head["clocks"],
+        "workloads": subs,
     }
     if rank == 0 and world == 1 and not args.skip_cpu:
-        rate, nch, tsec = cpu_oracle_rate(host0, 0, args.mode, args.cpu_seconds)
+        rate, nch, tsec = cpu_oracle_rate(head["host0"], 0, args.mode, args.cpu_seconds)
         line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": 1, "kind": "oracle",
                                 "sample": "%d chains of the %s batch through oracle.verify "
                                           "(numpy fp64, one thread), %.1f s"

@@ -152,6 +152,39 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
                   void *workspace, size_t workspace_bytes, sdv_stream_t stream);
 
 /*
+ * sdv_verify_pipelined - sdv_verify_ex for a stream of independent calls: the
+ * call may start streaming its window before the previous kernel on `stream` has
+ * finished, so that the latency-bound end of one call (the last chains' acceptance
+ * rule, U-draw and residual) overlaps the next call's read of its window.  The
+ * verification itself is the same (Algorithms block-verification, decomposition-res,
+ * u-sample); the results equal sdv_verify_ex's for the same arguments.
+ * Preconditions (the caller's promise; nothing checks them):
+ *   - the window (x_draft, mu_target, mu_draft, sigma, L_eff, mu_target_bonus,
+ *     sigma_bonus) is not written by earlier work on `stream` that may still be
+ *     running: the previous kernel, and the earlier calls of a run of pipelined
+ *     calls (the window is read while they finish);
+ *   - the workspace's counters are zero: the workspace is fresh from a
+ *     cudaMemset to 0, or was last used by a completed call of this library
+ *     (every call leaves them at zero).
+ * Outputs are written only after the previous kernel on `stream` has completed,
+ * so consecutive calls may share output buffers.  The overlap applies where a call
+ * is one kernel (B < 512 chains and rows of at most 16384 elements); other calls
+ * run exactly as sdv_verify_ex.  Same arguments, return codes and ownership as
+ * sdv_verify_ex; the workspace must not be shared with calls on other streams.
+ */
+int sdv_verify_pipelined(const void *x_draft, const void *mu_target, const void *mu_draft,
+                         const float *sigma, int64_t sigma_stride_b,
+                         int B, int L, int64_t d, int dtype,
+                         uint64_t seed, int mode,
+                         const int32_t *L_eff,
+                         const void *mu_target_bonus, const float *sigma_bonus,
+                         int residual_kind, float omega,
+                         int32_t *accepted_len, void *y_out,
+                         float *log_ratio_out, float *delta_norm_out, uint32_t *status_out,
+                         float *chain_aux_out,
+                         void *workspace, size_t workspace_bytes, sdv_stream_t stream);
+
+/*
  * sdv_verify_noalloc - sdv_verify without a workspace argument, for callers that
  * cannot allocate device memory.  (The paper has no counterpart; this is a
  * deployment option of this library.)  Such callers include plug-ins loaded into a
@@ -164,9 +197,11 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  *   - Returns SDV_ENOWORKSPACE, launching nothing, when
  *     sdv_workspace_bytes(B, L, d, dtype) > SDV_NOALLOC_SCRATCH_BYTES.
  *   - Calls no cudaMalloc / cudaFree or any other allocating routine.
- *   - The first call on a device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture on the device.
+ *   - Every call looks up the array's device address (cudaGetSymbolAddress) with
+ *     the caller's device current, so the address stays valid across a
+ *     cudaDeviceReset.  The first call on a device may also load the library's
+ *     device code there; make that first call before any stream capture on the
+ *     device.
  *   - Every call on a device shares the one array, which keeps the previous call's
  *     contents: the counters that must start at zero are cleared by each call on its
  *     own stream, but calls that overlap on the GPU (other streams, other host

@@ -49,8 +49,11 @@ def _sigma_args(sigma, Bn, L):
 
 def verify(x_draft, mu_target, mu_draft, sigma, seed, mode="block", *, L_eff=None,
            mu_target_bonus=None, sigma_bonus=None, residual="decomposition", omega=1.0,
-           with_ratios=True, with_aux=False, workspace=None, out=None):
-    """One verification call (sdv_verify_ex) on [B, L, d] CUDA tensors; returns a dict of outputs."""
+           with_ratios=True, with_aux=False, workspace=None, out=None, pipelined=False):
+    """One verification call (sdv_verify_ex) on [B, L, d] CUDA tensors; returns a dict of outputs.
+
+    pipelined=True calls sdv_verify_pipelined instead: the call may overlap the end of the
+    previous kernel on the stream (see its preconditions in include/specdiff.h)."""
     _need_cuda(x_draft, mu_target, mu_draft, sigma, L_eff, mu_target_bonus, sigma_bonus)
     Bn, L, d = x_draft.shape
     dt = x_draft.dtype
@@ -82,12 +85,13 @@ def verify(x_draft, mu_target, mu_draft, sigma, seed, mode="block", *, L_eff=Non
         aux = torch.empty(Bn, 4, dtype=torch.float32, device=dev) if aux is None else aux
     if workspace is None:
         workspace = make_workspace(Bn, L, d, dt, dev)
-    B.sdv_verify_ex(_ptr(x_draft), _ptr(mu_target), _ptr(mu_draft), _ptr(sigma), sstride,
-                    Bn, L, d, _DTYPES[dt], int(seed) & 0xFFFFFFFFFFFFFFFF, _MODES[mode],
-                    _ptr(L_eff), _ptr(mu_target_bonus), _ptr(sigma_bonus),
-                    _RESIDUALS[residual], float(omega),
-                    _ptr(acc), _ptr(y), _ptr(lr), _ptr(dn), _ptr(st), _ptr(aux),
-                    _ptr(workspace), workspace.numel(), _stream())
+    fn = B.sdv_verify_pipelined if pipelined else B.sdv_verify_ex
+    fn(_ptr(x_draft), _ptr(mu_target), _ptr(mu_draft), _ptr(sigma), sstride,
+       Bn, L, d, _DTYPES[dt], int(seed) & 0xFFFFFFFFFFFFFFFF, _MODES[mode],
+       _ptr(L_eff), _ptr(mu_target_bonus), _ptr(sigma_bonus),
+       _RESIDUALS[residual], float(omega),
+       _ptr(acc), _ptr(y), _ptr(lr), _ptr(dn), _ptr(st), _ptr(aux),
+       _ptr(workspace), workspace.numel(), _stream())
     res = dict(accepted_len=acc, y=y, status=st)
     if with_ratios:
         res.update(log_ratio=lr, delta_norm=dn)
@@ -117,6 +121,64 @@ def verify_host(x_draft, mu_target, mu_draft, sigma, seed, mode="block", *, dev_
     db["h_y"].copy_(db["y"], non_blocking=True)
     torch.cuda.current_stream().synchronize()
     return db["h_acc"], db["h_y"]
+
+
+class HostStream:
+    """End-to-end verification of a sequence of windows held in pinned host memory.
+
+    Each window is one pinned host tensor [3, B, L, d] (x_draft, mu_target, mu_draft
+    stacked, so that it crosses to the device in one copy) plus sigma.  ``depth`` device
+    slots are used in turn: the copy of a window into its slot (on a copy stream)
+    overlaps the verification of the previous one (on a compute stream), and each slot's
+    accepted lengths and states come back to pinned host memory on the compute stream.
+    ``submit`` returns the slot index; ``result`` waits for that slot and returns its
+    host tensors (valid until the slot is submitted again).  torch only allocates
+    memory and supplies the streams and events; the verification runs in libspecdiff.
+    """
+
+    def __init__(self, Bn, L, d, dtype=torch.float32, sigma_shape=None, depth=2, device="cuda"):
+        self.Bn, self.L, self.d, self.depth = Bn, L, d, depth
+        sigma_shape = (Bn, L) if sigma_shape is None else tuple(sigma_shape)
+        self.copy_stream = torch.cuda.Stream(device=device)
+        self.compute_stream = torch.cuda.Stream(device=device)
+        self.ws = torch.zeros(max(workspace_bytes(Bn, L, d, dtype), 256), dtype=torch.uint8, device=device)
+        self.slots = []
+        for _ in range(depth):
+            self.slots.append(dict(
+                win=torch.empty(3, Bn, L, d, dtype=dtype, device=device),
+                sigma=torch.empty(*sigma_shape, dtype=torch.float32, device=device),
+                accepted_len=torch.empty(Bn, dtype=torch.int32, device=device),
+                y=torch.empty(Bn, d, dtype=dtype, device=device),
+                status=torch.empty(Bn, dtype=torch.int32, device=device),
+                h_acc=torch.empty(Bn, dtype=torch.int32, pin_memory=True),
+                h_y=torch.empty(Bn, d, dtype=dtype, pin_memory=True),
+                copied=torch.cuda.Event(), done=torch.cuda.Event(), busy=False))
+        self.next = 0
+
+    def submit(self, window, sigma, seed, mode="block"):
+        i = self.next
+        self.next = (i + 1) % self.depth
+        sl = self.slots[i]
+        if sl["busy"]:
+            self.copy_stream.wait_event(sl["done"])      # the slot's previous window is verified
+        with torch.cuda.stream(self.copy_stream):
+            sl["win"].copy_(window, non_blocking=True)
+            sl["sigma"].copy_(sigma, non_blocking=True)
+            sl["copied"].record(self.copy_stream)
+        self.compute_stream.wait_event(sl["copied"])
+        with torch.cuda.stream(self.compute_stream):
+            w = sl["win"]
+            verify(w[0], w[1], w[2], sl["sigma"], seed, mode, with_ratios=False, workspace=self.ws, out=sl)
+            sl["h_acc"].copy_(sl["accepted_len"], non_blocking=True)
+            sl["h_y"].copy_(sl["y"], non_blocking=True)
+            sl["done"].record(self.compute_stream)
+        sl["busy"] = True
+        return i
+
+    def result(self, i):
+        sl = self.slots[i]
+        sl["done"].synchronize()
+        return sl["h_acc"], sl["h_y"]
 
 
 def make_device_buffers(Bn, L, d, dtype, sigma_shape, device="cuda"):

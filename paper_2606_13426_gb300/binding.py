@@ -51,6 +51,9 @@ SIGNATURES = {
     "sdv_verify_ex": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _U64, _I,
                            _P, _P, _P, _I, _F,
                            _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
+    "sdv_verify_pipelined": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _U64, _I,
+                                  _P, _P, _P, _I, _F,
+                                  _P, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "sdv_verify_noalloc": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _U64, _I,
                                 _P, _P, _P, _P, _P, _P]),
     "sdv_log_ratios": (_I, [_P, _P, _P, _P, _I64, _I, _I, _I64, _I, _P, _P, _P, _P, _SZ, _P]),
@@ -146,6 +149,16 @@ def sdv_verify_ex(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, 
                   chain_aux_out, workspace, workspace_bytes, stream):
     return _call("sdv_verify_ex", x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d,
                  dtype, seed, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+                 accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, chain_aux_out,
+                 workspace, workspace_bytes, stream)
+
+
+def sdv_verify_pipelined(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                         mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+                         accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
+                         chain_aux_out, workspace, workspace_bytes, stream):
+    return _call("sdv_verify_pipelined", x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L,
+                 d, dtype, seed, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
                  accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, chain_aux_out,
                  workspace, workspace_bytes, stream)
 

@@ -33,8 +33,14 @@ constexpr int64_t kK4MinChunk = 1024;
 constexpr int64_t kK4MaxChunk = 4096;
 constexpr int64_t kK4TargetCtas = 1024;
 // Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
-// finishes the chain inside the fused kernel; longer rows by k_resid_dot/_write.
-constexpr int64_t kFusedMaxGroups = 1024;
+// finishes the chain inside the fused kernel (the residual's noise cached in dynamic
+// shared memory: up to 64 KB, 3 resident CTAs per SM), kFinishMaxGroups on the
+// many-chain path (a static 16 KB cache in k_finish); longer rows by
+// k_resid_dot/_write.  The fused kernel's residual sweeps take kFusedResidUnroll
+// groups per thread, their loads issued together.
+constexpr int64_t kFusedMaxGroups = 4096;
+constexpr int64_t kFinishMaxGroups = 1024;
+constexpr int kFusedResidUnroll = 3;
 
 enum : int32_t {
   kKindInactive = 0,
@@ -98,15 +104,18 @@ struct WsLayout {
 WsLayout ws_layout(int B, int L, int64_t d, int dtype);
 
 // sdv_verify_ex with the seed taken from device memory when seed_dev is not null (it
-// is read by the kernels, so a captured call follows the value at replay), and event
-// timing skipped when timed is false.  Same validation and return codes.
+// is read by the kernels, so a captured call follows the value at replay), event
+// timing skipped when timed is false, and, with overlap, the permission to start
+// before the previous kernel on the stream has finished (sdv_verify_pipelined).  Same
+// validation and return codes.
 int verify_ex_impl(const void* x_draft, const void* mu_target, const void* mu_draft,
                    const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
                    uint64_t seed, const uint64_t* seed_dev, int mode, const int32_t* L_eff,
                    const void* mu_target_bonus, const float* sigma_bonus, int residual_kind,
                    float omega, int32_t* accepted_len, void* y_out, float* log_ratio_out,
                    float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
-                   void* workspace, size_t workspace_bytes, bool timed, void* stream);
+                   void* workspace, size_t workspace_bytes, bool timed, void* stream,
+                   bool overlap = false);
 
 // Records a cudaError_t for sdv_last_cuda_error() (this host thread).
 void set_last_cuda_error(int err);

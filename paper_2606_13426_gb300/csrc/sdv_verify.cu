@@ -212,40 +212,31 @@ __device__ __forceinline__ UParams shfl_params(const UParams& P, int src) {
   return R;
 }
 
-// For chain b: ell_j, |Delta_j| (from the tile partials, or given), coins and the
-// acceptance rule.  In block mode every candidate residual row j (lane j & 31 of
-// segment j >> 5) also gets the U-sampler setup at (|Delta_j|, log alpha_{j-1})
-// (log alpha_{-1} = 0), whose log v is the residual mass that h_{j-1} needs: the
-// scan evaluates it once for both.  Called by a full warp; every lane returns the
-// result.  Writes the per-chain outputs of ScanArgs except status and aux.
-__device__ ScanOut scan_warp(const ScanArgs& A, int b) {
+// Per-lane values of one chain's window, held by one warp: step j in lane j & 31 of
+// segment j >> 5 (L <= 64).
+struct ScanRegs {
+  float ell[2], dn[2], S1[2], S2[2], sg[2];
+  int g;         // window length gamma_k, clamped to [0, L]
+  bool any_bad;  // a non-finite ratio, norm or sigma
+};
+
+// Loads chain b's ell_j and |Delta_j|: from the tile partials (S1, S2 of every tile of
+// the row, read through L2) and sigma, or from given arrays.  Called by a full warp;
+// reads only.
+__device__ ScanRegs scan_load(const ScanArgs& A, int b) {
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int L = A.L;
+  ScanRegs R;
   // window length gamma_k, clamped to [0, L] (device data the host cannot check)
-  const int g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
-  if (g <= 0) {
-    if (lane == 0) {
-      if (A.accepted_len) A.accepted_len[b] = 0;
-      if (A.tau_out) A.tau_out[b] = 0;
-    }
-    if (A.ell_out)
-      for (int j = lane; j < L; j += 32) A.ell_out[(int64_t)b * L + j] = 0.f;
-    if (A.dn_out)
-      for (int j = lane; j < L; j += 32) A.dn_out[(int64_t)b * L + j] = 0.f;
-    ScanOut o;
-    o.cs = inactive_state();
-    o.have_P = false;
-    return o;
-  }
+  R.g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
   const int nseg = (L + 31) >> 5;
-  float ell[2], dn[2], S1[2], S2[2], sg[2];
   bool bad = false;
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
     const int j = lane + 32 * q;
-    ell[q] = 0.f; dn[q] = 0.f; S1[q] = 0.f; S2[q] = 0.f; sg[q] = 1.f;
-    if (q < nseg && j < g) {
+    R.ell[q] = 0.f; R.dn[q] = 0.f; R.S1[q] = 0.f; R.S2[q] = 0.f; R.sg[q] = 1.f;
+    if (q < nseg && j < R.g) {
       if (A.part) {
         // partials written by other CTAs of this grid: read through L2
         const float2* p = A.part + ((int64_t)b * L + j) * A.C;
@@ -257,28 +248,61 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
           a2 += t.y;
         }
         const float s = A.sigma[(int64_t)b * A.sstride + j];
-        S1[q] = a1; S2[q] = a2; sg[q] = s;
-        ell[q] = -(a1 + 0.5f * a2) / (s * s);
-        dn[q] = sqrtf(a2) / s;
+        R.S1[q] = a1; R.S2[q] = a2; R.sg[q] = s;
+        R.ell[q] = -(a1 + 0.5f * a2) / (s * s);
+        R.dn[q] = sqrtf(a2) / s;
         if (!(s > 0.f) || !isfinite(s)) bad = true;
       } else {
-        ell[q] = A.ell_in[(int64_t)b * L + j];
-        dn[q] = A.dn_in[(int64_t)b * L + j];
+        R.ell[q] = A.ell_in[(int64_t)b * L + j];
+        R.dn[q] = A.dn_in[(int64_t)b * L + j];
       }
-      if (!isfinite(ell[q]) || !isfinite(dn[q])) bad = true;
-    }
-    if (q < nseg && j < L) {
-      if (A.ell_out) A.ell_out[(int64_t)b * L + j] = ell[q];
-      if (A.dn_out) A.dn_out[(int64_t)b * L + j] = dn[q];
+      if (!isfinite(R.ell[q]) || !isfinite(R.dn[q])) bad = true;
     }
   }
-  const bool any_bad = __any_sync(FULL, bad);
+  R.any_bad = __any_sync(FULL, bad);
+  return R;
+}
+
+// The per-step outputs (ell_j, |Delta_j|; zero outside the window) by the lanes of the warp
+// that loaded R.
+__device__ __forceinline__ void scan_write_steps(const ScanArgs& A, int b, const ScanRegs& R) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int j = lane + 32 * q;
+    if (j < A.L) {
+      if (A.ell_out) A.ell_out[(int64_t)b * A.L + j] = R.ell[q];
+      if (A.dn_out) A.dn_out[(int64_t)b * A.L + j] = R.dn[q];
+    }
+  }
+}
+
+// The per-chain outputs known after the acceptance rule (accepted length, tau, log
+// alpha_res), by one thread.
+__device__ __forceinline__ void scan_write_chain(const ScanArgs& A, int b, const ChainState& cs) {
+  if (A.ratios_only) return;
+  if (A.accepted_len) A.accepted_len[b] = cs.tau > 0 ? cs.tau - 1 : 0;
+  if (A.tau_out) A.tau_out[b] = cs.tau;
+  if (A.la_res_out && cs.kind != kKindInactive) A.la_res_out[b] = cs.la_res;
+}
+
+// For chain b with loaded values R: coins and the acceptance rule.  In block mode every
+// candidate residual row j (lane j & 31 of segment j >> 5) also gets the U-sampler setup
+// at (|Delta_j|, log alpha_{j-1}) (log alpha_{-1} = 0), whose log v is the residual mass
+// that h_{j-1} needs: the scan evaluates it once for both.  Called by a full warp; every
+// lane returns the result.  Writes nothing.
+__device__ ScanOut scan_decide(const ScanArgs& A, int b, const ScanRegs& R) {
+  const unsigned FULL = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int L = A.L;
+  const int g = R.g;
   ScanOut out;
   out.have_P = false;
-  if (A.ratios_only) {
+  if (g <= 0 || A.ratios_only) {
     out.cs = inactive_state();
     return out;
   }
+  const int nseg = (L + 31) >> 5;
 
   // coins: eta_j from Philox (b, j, 0, 0), word 0, compared in log space
   float leta[2];
@@ -289,7 +313,7 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
     if (q < nseg && j < g)
       leta[q] = log_uniform(philox_block(seed_of(A), (uint32_t)b, (uint32_t)j, kStreamCoin, 0u).x);
   }
-  const float ellw[2] = {ell[0] * A.inv_omega2, ell[1] * A.inv_omega2};
+  const float ellw[2] = {R.ell[0] * A.inv_omega2, R.ell[1] * A.inv_omega2};
 
   int tau;             // 1-based
   float la_res = 0.f;  // log alpha_{tau-1}
@@ -330,16 +354,16 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
       if (q < nseg) {  // warp-uniform
-        const bool ok = (dn[q] > 0.f) && isfinite(dn[q]) && isfinite(lap[q]);
-        Pq[q] = usample_setup(ok ? dn[q] : 1.f, ok ? fminf(lap[q], 0.f) : -1.f);
+        const bool ok = (R.dn[q] > 0.f) && isfinite(R.dn[q]) && isfinite(lap[q]);
+        Pq[q] = usample_setup(ok ? R.dn[q] : 1.f, ok ? fminf(lap[q], 0.f) : -1.f);
       } else {
         Pq[q] = UParams{};
       }
     }
     // h_j (0-based j) uses |Delta| and log v of step j + 1 (the paper's D_{j+1})
-    const float dnx0 = __shfl_down_sync(FULL, dn[0], 1);
-    const float dnx1 = __shfl_down_sync(FULL, dn[1], 1);
-    const float dnf1 = __shfl_sync(FULL, dn[1], 0);
+    const float dnx0 = __shfl_down_sync(FULL, R.dn[0], 1);
+    const float dnx1 = __shfl_down_sync(FULL, R.dn[1], 1);
+    const float dnf1 = __shfl_sync(FULL, R.dn[1], 0);
     const float lvx0 = __shfl_down_sync(FULL, Pq[0].lv, 1);
     const float lvx1 = __shfl_down_sync(FULL, Pq[1].lv, 1);
     const float lvf1 = __shfl_sync(FULL, Pq[1].lv, 0);
@@ -384,12 +408,12 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
   const bool resid = tau <= g;
   const int rrow = resid ? tau - 1 : 0;
   const int rq = rrow >> 5, rl = rrow & 31;
-  const float Dt = rq ? __shfl_sync(FULL, dn[1], rl) : __shfl_sync(FULL, dn[0], rl);
-  const float st = rq ? __shfl_sync(FULL, sg[1], rl) : __shfl_sync(FULL, sg[0], rl);
-  const float S1t = rq ? __shfl_sync(FULL, S1[1], rl) : __shfl_sync(FULL, S1[0], rl);
-  const float S2t = rq ? __shfl_sync(FULL, S2[1], rl) : __shfl_sync(FULL, S2[0], rl);
+  const float Dt = rq ? __shfl_sync(FULL, R.dn[1], rl) : __shfl_sync(FULL, R.dn[0], rl);
+  const float st = rq ? __shfl_sync(FULL, R.sg[1], rl) : __shfl_sync(FULL, R.sg[0], rl);
+  const float S1t = rq ? __shfl_sync(FULL, R.S1[1], rl) : __shfl_sync(FULL, R.S1[0], rl);
+  const float S2t = rq ? __shfl_sync(FULL, R.S2[1], rl) : __shfl_sync(FULL, R.S2[0], rl);
 
-  uint32_t status = any_bad ? 2u : 0u;
+  uint32_t status = R.any_bad ? 2u : 0u;
   int kind;
   if (!resid) {
     kind = A.has_bonus ? kKindBonus : kKindCopy;
@@ -400,11 +424,6 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
     kind = kKindReflect;
   } else {
     kind = kKindResid;
-  }
-  if (lane == 0) {
-    if (A.accepted_len) A.accepted_len[b] = tau - 1;
-    if (A.tau_out) A.tau_out[b] = tau;
-    if (A.la_res_out) A.la_res_out[b] = la_res;
   }
   ChainState& cs = out.cs;
   cs.tau = tau;
@@ -419,6 +438,16 @@ __device__ ScanOut scan_warp(const ScanArgs& A, int b) {
   cs.kind = kind;
   cs.pad[0] = cs.pad[1] = 0;
   return out;
+}
+
+// scan_load, the per-step outputs, scan_decide and the per-chain outputs in one go (the
+// kernels whose writes need not wait for an earlier grid).
+__device__ ScanOut scan_warp(const ScanArgs& A, int b) {
+  const ScanRegs R = scan_load(A, b);
+  scan_write_steps(A, b, R);
+  const ScanOut o = scan_decide(A, b, R);
+  if ((threadIdx.x & 31) == 0) scan_write_chain(A, b, o.cs);
+  return o;
 }
 
 // Per-chain outputs that depend on U: status bits and (U, log alpha_res, |Delta_tau|,
@@ -436,11 +465,10 @@ __device__ __forceinline__ void report_chain(const ScanArgs& A, int b, const Cha
   }
 }
 
-// Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch), then
-// the chain's reported outputs.
+// Residual 1-D draw of a finished chain by the whole CTA (CTA-uniform branch).
 template <int NT>
-__device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, ChainState& cs,
-                                                  const UParams* P, USampleScratch* us) {
+__device__ __forceinline__ void draw_u(const ScanArgs& A, int b, ChainState& cs, const UParams* P,
+                                       USampleScratch* us) {
   if (cs.kind == kKindResid && A.draw_u) {
     const uint32_t wbits = philox_block(seed_of(A), (uint32_t)b, 0u, kStreamUSample, 0u).x;
     uint32_t st = cs.status;
@@ -448,7 +476,17 @@ __device__ __forceinline__ void draw_u_and_report(const ScanArgs& A, int b, Chai
     cs.U = usample_block<NT>(Q, wbits, &st, us);
     cs.status = st;
   }
-  report_chain(A, b, cs, threadIdx.x == 0);
+}
+
+// Grid dependencies (programmatic dependent launch).  A kernel launched with the
+// programmatic-serialisation attribute may start while the previous kernel on its
+// stream is still running, as soon as every CTA of that kernel has called
+// griddep_launch_dependents or exited; griddep_wait blocks until the previous kernel has
+// completed and its writes are visible.  Without that attribute (or with no previous
+// kernel) both are no-ops.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // ---------------------------------------------------------------- residual row
@@ -476,20 +514,56 @@ struct CtaGroup {
   }
 };
 
-// Writes y[b, :] for chain state cs with the threads of group grp (every thread of
-// the group calls it with the same cs).  Decomposition: pass A reduces delta^T G,
-// pass B writes m^q + sigma (G + e (U - e^T G)).  With gcache (room for the row's
-// groups, used only by the thread that owns a group) pass A keeps G there for pass
-// B (GMODE 1), or the caller has filled it already (GMODE 2: drawn by warps that
-// would otherwise wait on the scan); with GMODE 0 pass B draws G again (same
-// Philox counters).  Each thread handles RU
-// groups of four elements per sweep, the loads of all of them issued before any use.
+// The decomposition residual's coefficient U - e^T G of chain state cs (pass A: reduces
+// delta^T G over the rejected row with the threads of group grp, every thread of the
+// group calling it with the same cs; 0 for the other kinds).  With gcache (room for the
+// row's groups, each used only by the thread that owns the group) pass A keeps G there
+// for pass B (GMODE 1), or the caller has filled it already (GMODE 2: drawn by warps that
+// would otherwise wait on the scan); with GMODE 0 pass B draws G again (same Philox
+// counters).  Each thread handles RU groups of four elements per sweep, the loads of all
+// of them issued before any use.  Reads only (and gcache with GMODE 1).
 template <typename T, bool VEC4, int RU, int GMODE, typename Group>
-__device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
-                             const T* __restrict__ mp, const T* __restrict__ mq_bonus,
-                             const float* __restrict__ sigma_bonus, int L, int64_t d,
-                             uint64_t seed, int b, const ChainState& cs, T* __restrict__ y,
-                             const Group& grp, float4* gcache) {
+__device__ float residual_coef(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d,
+                               uint64_t seed, int b, const ChainState& cs, const Group& grp,
+                               float4* gcache) {
+  if (cs.kind != kKindResid) return 0.f;
+  const int nt = grp.size();
+  const int64_t ng = (d + 3) / 4;
+  const int64_t rbase = ((int64_t)b * L + cs.row) * d;
+  // groups past the row end load zeros (load4 guards each element)
+  float sp = 0.f;
+  for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
+    float fq[RU][4], fp[RU][4];
+#pragma unroll
+    for (int u = 0; u < RU; ++u) {
+      load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
+      load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < RU; ++u) {
+      const int64_t gi = g0 + (int64_t)u * nt;
+      const float4 G = (GMODE == 2) ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
+                                    : normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
+      if (GMODE == 1 && gi < ng) gcache[gi] = G;
+      sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
+      sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
+      sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
+      sp = fmaf(fp[u][3] - fq[u][3], G.w, sp);
+    }
+  }
+  return cs.U - grp.all_sum(sp) * cs.inv_norm;  // U - e^T G
+}
+
+// Writes y[b, :] for chain state cs with the threads of group grp (pass B): the
+// decomposition residual m^q + sigma (G + e coef) with coef from residual_coef, the
+// reflection x - delta (1 + 2 S1/S2), m^q + sigma G for a zero shift, the bonus step,
+// or the last accepted draft.
+template <typename T, bool VEC4, int RU, int GMODE, typename Group>
+__device__ void residual_write(const T* __restrict__ x, const T* __restrict__ mq,
+                               const T* __restrict__ mp, const T* __restrict__ mq_bonus,
+                               const float* __restrict__ sigma_bonus, int L, int64_t d,
+                               uint64_t seed, int b, const ChainState& cs, float coef,
+                               T* __restrict__ y, const Group& grp, const float4* gcache) {
   if (cs.kind == kKindInactive) return;
   const int nt = grp.size();
   const int64_t ng = (d + 3) / 4;
@@ -497,27 +571,6 @@ __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
   const int64_t ybase = (int64_t)b * d;
   // groups past the row end load zeros (load4 guards each element) and store nothing
   if (cs.kind == kKindResid) {
-    float sp = 0.f;
-    for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
-      float fq[RU][4], fp[RU][4];
-#pragma unroll
-      for (int u = 0; u < RU; ++u) {
-        load4<T, VEC4>(mq + rbase, 4 * (g0 + (int64_t)u * nt), d, fq[u]);
-        load4<T, VEC4>(mp + rbase, 4 * (g0 + (int64_t)u * nt), d, fp[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < RU; ++u) {
-        const int64_t gi = g0 + (int64_t)u * nt;
-        const float4 G = (GMODE == 2) ? (gi < ng ? gcache[gi] : make_float4(0.f, 0.f, 0.f, 0.f))
-                                      : normals4_f(seed, (uint32_t)b, (uint32_t)gi, kStreamResid, 0u);
-        if (GMODE == 1 && gi < ng) gcache[gi] = G;
-        sp = fmaf(fp[u][0] - fq[u][0], G.x, sp);  // tail elements load 0 and contribute 0
-        sp = fmaf(fp[u][1] - fq[u][1], G.y, sp);
-        sp = fmaf(fp[u][2] - fq[u][2], G.z, sp);
-        sp = fmaf(fp[u][3] - fq[u][3], G.w, sp);
-      }
-    }
-    const float coef = cs.U - grp.all_sum(sp) * cs.inv_norm;  // U - e^T G
     for (int64_t g0 = grp.rank(); g0 < ng; g0 += (int64_t)nt * RU) {
       float fq[RU][4], fp[RU][4];
 #pragma unroll
@@ -580,6 +633,17 @@ __device__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
   }
 }
 
+// Both passes (the writers that need not wait for an earlier grid in between).
+template <typename T, bool VEC4, int RU, int GMODE, typename Group>
+__device__ __forceinline__ void residual_row(const T* __restrict__ x, const T* __restrict__ mq,
+                                             const T* __restrict__ mp, const T* __restrict__ mq_bonus,
+                                             const float* __restrict__ sigma_bonus, int L, int64_t d,
+                                             uint64_t seed, int b, const ChainState& cs,
+                                             T* __restrict__ y, const Group& grp, float4* gcache) {
+  const float coef = residual_coef<T, VEC4, RU, GMODE>(mq, mp, L, d, seed, b, cs, grp, gcache);
+  residual_write<T, VEC4, RU, GMODE>(x, mq, mp, mq_bonus, sigma_bonus, L, d, seed, b, cs, coef, y, grp, gcache);
+}
+
 // The residual's G of chain b (stream kStreamResid) for groups [first, ng), every
 // `step`-th group, into gcache: drawn by the finishing CTA's warps other than the
 // scanning warp, before the rejected step is known (G does not depend on it).
@@ -604,8 +668,27 @@ struct VerifyArgs {
   ScanArgs S;
 };
 
-// RESID: 1 = this kernel writes y; 0 = it leaves the chain state for k_resid_*.
-template <typename T, bool VEC, int VPT, bool VEC4, int RESID>
+// Fetch-and-increment of chain b's ticket with acquire-release semantics at GPU scope,
+// wrapping to 0 after `last` (atom.inc: old >= last ? 0 : old + 1): the CTA that draws
+// `last` holds the chain's last tile, and the counter is back at 0 for the next call.
+// The release publishes this CTA's partial; the holder of the last ticket acquires
+// every partial released before it.
+__device__ __forceinline__ unsigned int ticket_inc(unsigned int* p, unsigned int last) {
+  unsigned int old;
+  asm volatile("atom.acq_rel.gpu.global.inc.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(last) : "memory");
+  return old;
+}
+
+// RESID: 1 = this kernel writes y (the residual's G cached in dynamic shared memory,
+// (d + 3)/4 float4); 0 = it leaves the chain state for k_resid_*.  RU: groups of four
+// elements per thread per residual sweep.
+//
+// Ordering against the previous kernel on the stream (see griddep_wait): this kernel
+// writes nothing the previous one may read except its own outputs, and those only after
+// griddep_wait; a finishing CTA triggers its dependents once it has read the chain's
+// partials, the only workspace data that the next call overwrites; the tickets return
+// to zero by themselves.  So consecutive calls may overlap when the caller allows it.
+template <typename T, bool VEC, int VPT, bool VEC4, int RESID, int RU>
 __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs A) {
   __shared__ float2 red[kK1Threads / 32];
   __shared__ int last_s;
@@ -614,7 +697,8 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   __shared__ UParams P_s;
   __shared__ bool haveP_s;
   __shared__ USampleScratch us;
-  __shared__ float4 g_s[RESID ? kFusedMaxGroups : 1];  // the residual's G, drawn once
+  __shared__ float ell_s[SDV_MAX_L], dn_s[SDV_MAX_L];
+  extern __shared__ float4 g_s[];  // RESID: the residual's G, drawn once
   const int L = A.S.L;
   const int C = A.S.C;
   const int64_t tile = blockIdx.x;
@@ -628,6 +712,7 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   if (g == 0) {
     // inactive chain: tile (b, 0, 0) writes its outputs, nothing is streamed
     if (j == 0 && c == 0 && threadIdx.x < 32) {
+      griddep_wait();
       const ChainState cs = scan_warp(A.S, b).cs;
       if (threadIdx.x == 0 && RESID == 0) A.state[b] = cs;
     }
@@ -640,33 +725,60 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
   const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
   if (threadIdx.x == 0) {
     A.part[tile] = t;
-    // release this partial with the ticket; the chain's last ticket also acquires
-    // every partial released before it (one acq_rel atomic instead of two fences)
-    const unsigned int k = ticket_acq_rel(A.ticket + b);
-    last_s = (k == (unsigned int)(g * C) - 1u);
+    const unsigned int last = (unsigned int)(g * C) - 1u;
+    last_s = (ticket_inc(A.ticket + b, last) == last);
   }
   __syncthreads();  // thread 0's acquire reaches warp 0's partial loads through the barrier
   if (!last_s) return;
+  ScanRegs R;
   if (threadIdx.x < 32) {
-    const ScanOut so = scan_warp(A.S, b);
+    R = scan_load(A.S, b);
+    const int lane = threadIdx.x;
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      if (lane + 32 * q < L) {
+        ell_s[lane + 32 * q] = R.ell[q];
+        dn_s[lane + 32 * q] = R.dn[q];
+      }
+    }
+  }
+  __syncthreads();
+  griddep_launch_dependents();  // this chain's partials are read
+  if (A.S.ratios_only) {
+    griddep_wait();
+    if (threadIdx.x < 32) scan_write_steps(A.S, b, R);
+    return;
+  }
+  if (threadIdx.x < 32) {
+    const ScanOut so = scan_decide(A.S, b, R);
     if (threadIdx.x == 0) {
       cs_s = so.cs;
       P_s = so.P;
       haveP_s = so.have_P;
     }
-  } else if (RESID && !A.S.ratios_only) {
+  } else if (RESID) {
     prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, kK1Threads - 32, g_s);
   }
   __syncthreads();
-  if (A.S.ratios_only) return;
   ChainState cs = cs_s;
-  draw_u_and_report<kK1Threads>(A.S, b, cs, haveP_s ? &P_s : nullptr, &us);
-  if (RESID == 0) {
-    if (threadIdx.x == 0) A.state[b] = cs;
-  } else {
-    residual_row<T, VEC4, 1, 2>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S),
-                                b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
+  draw_u<kK1Threads>(A.S, b, cs, haveP_s ? &P_s : nullptr, &us);
+  const CtaGroup grp{red, &bcast};
+  float coef = 0.f;
+  if (RESID) coef = residual_coef<T, VEC4, RU, 2>(mq, mp, L, A.d, seed_of(A.S), b, cs, grp, g_s);
+  // every write of this call's outputs comes after the previous kernel has completed
+  griddep_wait();
+  for (int i = threadIdx.x; i < L; i += kK1Threads) {
+    if (A.S.ell_out) A.S.ell_out[(int64_t)b * L + i] = ell_s[i];
+    if (A.S.dn_out) A.S.dn_out[(int64_t)b * L + i] = dn_s[i];
   }
+  if (threadIdx.x == 0) {
+    scan_write_chain(A.S, b, cs);
+    report_chain(A.S, b, cs, true);
+    if (RESID == 0) A.state[b] = cs;
+  }
+  if (RESID)
+    residual_write<T, VEC4, RU, 2>(x, mq, mp, (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S), b, cs,
+                                   coef, (T*)A.y, grp, g_s);
 }
 
 // ---------------------------------------------------------------- many-chain path
@@ -703,7 +815,7 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
   __shared__ ChainState cs_s;
   __shared__ float2 red[kFinishThreads / 32];
   __shared__ float bcast;
-  __shared__ float4 g_s[RESID ? kFusedMaxGroups : 1];  // the residual's G, drawn once
+  __shared__ float4 g_s[RESID ? kFinishMaxGroups : 1];  // the residual's G, drawn once
   const int b = blockIdx.x;
   if (threadIdx.x < 32) {
     const ScanOut so = scan_warp(A.S, b);
@@ -960,34 +1072,57 @@ static int validate_window(const void* x, const void* mq, const void* mp, const 
   return SDV_OK;
 }
 
+// One launch of k_verify: dynamic shared memory for the residual's noise cache (RESID),
+// and, with `overlap`, the programmatic-serialisation attribute that lets the kernel
+// start before the previous kernel on the stream has finished.
+template <typename Kern>
+static cudaError_t launch_k1(Kern kern, unsigned tiles, size_t smem, bool overlap, const VerifyArgs& A,
+                             cudaStream_t s) {
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(tiles);
+  cfg.blockDim = dim3(kK1Threads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = overlap ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, A);
+}
+
 template <typename T, int RESID>
-static void launch_verify(const VerifyArgs& A, int B, int L, int vpt, cudaStream_t s) {
+static cudaError_t launch_verify(const VerifyArgs& A, int B, int L, int vpt, bool overlap, cudaStream_t s) {
   constexpr int V = 16 / (int)sizeof(T);
+  constexpr int RU = RESID ? kFusedResidUnroll : 1;
   const bool vec = (A.d % V == 0) && aligned(A.x, 16) && aligned(A.mq, 16) && aligned(A.mp, 16);
   const bool vec4 = (A.d % 4 == 0) && aligned(A.x, 4 * sizeof(T)) && aligned(A.mq, 4 * sizeof(T)) &&
                     aligned(A.mp, 4 * sizeof(T)) && (A.y == nullptr || aligned(A.y, 4 * sizeof(T))) &&
                     (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
   const unsigned tiles = (unsigned)((int64_t)B * L * A.S.C);
-#define SDV_LAUNCH(VECV, VPTV, V4) k_verify<T, VECV, VPTV, V4, RESID><<<tiles, kK1Threads, 0, s>>>(A)
+  const size_t smem = (RESID && !A.S.ratios_only) ? sizeof(float4) * (size_t)((A.d + 3) / 4) : 0;
+#define SDV_LAUNCH(VECV, VPTV, V4) return launch_k1(k_verify<T, VECV, VPTV, V4, RESID, RU>, tiles, smem, overlap, A, s)
   if (!vec) {
     if (vec4) SDV_LAUNCH(false, 1, true);
-    else SDV_LAUNCH(false, 1, false);
-    return;
+    SDV_LAUNCH(false, 1, false);
   }
   if (vec4) {
     switch (vpt) {
-      case 1: SDV_LAUNCH(true, 1, true); break;
-      case 2: SDV_LAUNCH(true, 2, true); break;
-      case 3: SDV_LAUNCH(true, 3, true); break;
-      default: SDV_LAUNCH(true, 4, true); break;
+      case 1: SDV_LAUNCH(true, 1, true);
+      case 2: SDV_LAUNCH(true, 2, true);
+      case 3: SDV_LAUNCH(true, 3, true);
+      default: SDV_LAUNCH(true, 4, true);
     }
-  } else {
-    switch (vpt) {
-      case 1: SDV_LAUNCH(true, 1, false); break;
-      case 2: SDV_LAUNCH(true, 2, false); break;
-      case 3: SDV_LAUNCH(true, 3, false); break;
-      default: SDV_LAUNCH(true, 4, false); break;
-    }
+  }
+  switch (vpt) {
+    case 1: SDV_LAUNCH(true, 1, false);
+    case 2: SDV_LAUNCH(true, 2, false);
+    case 3: SDV_LAUNCH(true, 3, false);
+    default: SDV_LAUNCH(true, 4, false);
   }
 #undef SDV_LAUNCH
 }
@@ -1046,8 +1181,8 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
                           const void* mu_target_bonus, const float* sigma_bonus,
                           int residual_kind, float omega, int32_t* accepted_len, void* y_out,
                           float* log_ratio_out, float* delta_norm_out, uint32_t* status_out,
-                          float* chain_aux_out, bool ratios_only, bool timed, void* workspace,
-                          cudaStream_t s) {
+                          float* chain_aux_out, bool ratios_only, bool timed, bool overlap,
+                          void* workspace, cudaStream_t s) {
   const WsLayout w = ws_layout(B, L, d, dtype);
   char* ws = (char*)workspace;
   VerifyArgs A{};
@@ -1067,24 +1202,36 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
 
   cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
-  const bool long_rows = (d + 3) / 4 > kFusedMaxGroups;
   const bool many = !ratios_only && B >= kManyChainMin;
+  // rows whose residual the finishing CTA writes itself (k_verify: its noise cache in
+  // dynamic shared memory; k_finish: a static cache); longer rows go to k_resid_*
+  const bool long_rows = !ratios_only && (d + 3) / 4 > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
+  // consecutive calls may overlap only on the single-kernel path
+  overlap = overlap && !many && !long_rows;
+  cudaError_t e = cudaSuccess;
   if (many) {
     if (f32) launch_tiles<float>(A, B, L, w.vpt1, s);
     else launch_tiles<__nv_bfloat16>(A, B, L, w.vpt1, s);
   } else {
-    if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+    // the tickets return to zero at the end of every call; a call that may overlap
+    // its predecessor relies on that (the caller's contract), the others clear them
+    if (!overlap && cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
       check_launch();
       return SDV_ECUDA;
     }
-    if (long_rows && !ratios_only) {
-      if (f32) launch_verify<float, 0>(A, B, L, w.vpt1, s);
-      else launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, s);
+    if (long_rows) {
+      e = f32 ? launch_verify<float, 0>(A, B, L, w.vpt1, false, s)
+              : launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, false, s);
     } else {
-      if (f32) launch_verify<float, 1>(A, B, L, w.vpt1, s);
-      else launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, s);
+      e = f32 ? launch_verify<float, 1>(A, B, L, w.vpt1, overlap, s)
+              : launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, overlap, s);
     }
+  }
+  if (e != cudaSuccess) {
+    g_last_cuda_error = (int)e;
+    cudaGetLastError();
+    return SDV_ECUDA;
   }
   int rc = check_launch();
   if (rc != SDV_OK) return rc;
@@ -1099,7 +1246,7 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
     }
     if ((rc = check_launch()) != SDV_OK) return rc;
   }
-  if (long_rows && !ratios_only) {
+  if (long_rows) {
     float* part4 = (float*)(ws + w.part4_off);
     if (f32)
       launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev, w, A.state, part4, y_out, s);
@@ -1117,7 +1264,7 @@ int verify_ex_impl(const void* x_draft, const void* mu_target, const void* mu_dr
                         const void* mu_target_bonus, const float* sigma_bonus, int residual_kind,
                         float omega, int32_t* accepted_len, void* y_out, float* log_ratio_out,
                         float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
-                        void* workspace, size_t workspace_bytes, bool timed, void* stream) {
+                        void* workspace, size_t workspace_bytes, bool timed, void* stream, bool overlap) {
   int rc = validate_window(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype);
   if (rc != SDV_OK) return rc;
   if (mode != SDV_MODE_SAMPLE && mode != SDV_MODE_BLOCK) return SDV_EINVAL;
@@ -1140,7 +1287,7 @@ int verify_ex_impl(const void* x_draft, const void* mu_target, const void* mu_dr
   return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
                         seed_dev, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
                         accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
-                        chain_aux_out, false, timed, workspace, (cudaStream_t)stream);
+                        chain_aux_out, false, timed, overlap, workspace, (cudaStream_t)stream);
 }
 
 }  // namespace sdv
@@ -1179,7 +1326,20 @@ int sdv_verify_ex(const void* x_draft, const void* mu_target, const void* mu_dra
   return verify_ex_impl(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
                         nullptr, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
                         accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
-                        chain_aux_out, workspace, workspace_bytes, true, stream);
+                        chain_aux_out, workspace, workspace_bytes, true, stream, false);
+}
+
+int sdv_verify_pipelined(const void* x_draft, const void* mu_target, const void* mu_draft,
+                         const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d, int dtype,
+                         uint64_t seed, int mode, const int32_t* L_eff, const void* mu_target_bonus,
+                         const float* sigma_bonus, int residual_kind, float omega,
+                         int32_t* accepted_len, void* y_out, float* log_ratio_out,
+                         float* delta_norm_out, uint32_t* status_out, float* chain_aux_out,
+                         void* workspace, size_t workspace_bytes, sdv_stream_t stream) {
+  return verify_ex_impl(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed,
+                        nullptr, mode, L_eff, mu_target_bonus, sigma_bonus, residual_kind, omega,
+                        accepted_len, y_out, log_ratio_out, delta_norm_out, status_out,
+                        chain_aux_out, workspace, workspace_bytes, true, stream, true);
 }
 
 int sdv_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
@@ -1208,7 +1368,7 @@ int sdv_log_ratios(const void* x_draft, const void* mu_target, const void* mu_dr
   return enqueue_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, 0,
                         nullptr, SDV_MODE_BLOCK, L_eff, nullptr, nullptr, SDV_RESIDUAL_DECOMPOSITION,
                         1.0f, nullptr, nullptr, log_ratio_out, delta_norm_out, nullptr, nullptr, true,
-                        false, workspace, (cudaStream_t)stream);
+                        false, false, workspace, (cudaStream_t)stream);
 }
 
 int sdv_accept_scan(const float* log_ratio, const float* delta_norm, int B, int L,

@@ -1,5 +1,5 @@
 """bench.py's host-side accounting, checked on the CPU: launches per call, algorithmic
-bytes of the first kernel, the shared workload name of both arms, and the lookup of a
+bytes of a call, the shared workload name of both arms, and the lookup of a
 profile's traffic (only for the workload's full batch and a matching source hash)."""
 import os
 import re
@@ -14,18 +14,17 @@ class _Args:
 
 
 def test_launches_per_call():
-    assert bench.launches_per_step(256, 3072) == 1      # fused kernel (tickets reset by a memset)
-    assert bench.launches_per_step(64, 16384) == 3      # + long-row dot and write
+    assert bench.launches_per_step(256, 3072) == 1      # fused kernel
+    assert bench.launches_per_step(64, 16384) == 1      # rows up to 16384 elements stay fused
+    assert bench.launches_per_step(16, 196608) == 3     # + long-row dot and write
     assert bench.launches_per_step(1024, 3072) == 2     # k_tiles + k_finish
-    assert bench.launches_per_step(1024, 16384) == 4
+    assert bench.launches_per_step(1024, 16384) == 4    # k_finish caches up to 4096 elements
 
 
-def test_algorithmic_bytes_of_the_first_kernel():
-    # pixel: window + rejected rows (read m^q, m^p) + y, all fp32
-    assert bench.fused_kernel_bytes(256, 8, 3072, "f32") == 3 * 256 * 8 * 3072 * 4 + 3 * 256 * 3072 * 4
-    # long rows and the many-chain streaming kernel move the window alone
-    assert bench.fused_kernel_bytes(64, 16, 16384, "bf16") == 3 * 64 * 16 * 16384 * 2
-    assert bench.fused_kernel_bytes(1024, 8, 3072, "f32") == 3 * 1024 * 8 * 3072 * 4
+def test_algorithmic_bytes_of_a_call():
+    # window read once, plus the rejected rows (m^q, m^p re-read) and y written, per chain
+    assert bench.call_bytes(256, 8, 3072, "f32") == 3 * 256 * 8 * 3072 * 4 + 3 * 256 * 3072 * 4
+    assert bench.call_bytes(64, 16, 16384, "bf16") == 3 * 64 * 16 * 16384 * 2 + 3 * 64 * 16384 * 2
 
 
 def test_both_arms_name_the_workload_alike():
@@ -44,4 +43,4 @@ def test_profile_traffic_lookup():
     assert bench.profile_traffic("tiny", True) is None       # no summary for this workload
     # traffic, when reported, is the window plus at most the rejected rows and y
     if got is not None:
-        assert 3 * 256 * 8 * 3072 * 4 <= got <= 1.02 * bench.fused_kernel_bytes(256, 8, 3072, "f32")
+        assert 3 * 256 * 8 * 3072 * 4 <= got <= 1.02 * bench.call_bytes(256, 8, 3072, "f32")

@@ -1,0 +1,119 @@
+"""sdv_verify_pipelined: runs of independent verification calls whose kernels may overlap
+on one stream (each call starts streaming its window while the previous call's last
+chains finish).  The kernels are those of sdv_verify_ex, so every call's outputs must
+equal, bit for bit, those of a plain call on the same inputs (which the other GPU tests
+compare with the oracle) -- with separate outputs per call, with outputs shared by all
+calls (written in call order), and under CUDA-graph capture."""
+import numpy as np
+import pytest
+import torch
+
+import workloads as W
+from gpu_helpers import to_dev
+
+pytestmark = pytest.mark.gpu
+
+KEYS = ("accepted_len", "y", "status", "log_ratio", "delta_norm", "aux")
+
+
+@pytest.fixture(scope="module")
+def api():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2606_13426_gb300 import api as A
+    return A
+
+
+def _sets(kind, n, B, L, d, ragged):
+    out = []
+    for i in range(n):
+        inp = W.make_verify_inputs(kind, B=B, L=L, d=d, seed=50 + i, per_chain_sigma=True)
+        s = dict(x=to_dev(inp, "x_draft"), mq=to_dev(inp, "mu_target"), mp=to_dev(inp, "mu_draft"),
+                 sigma=torch.from_numpy(inp["sigma"]).cuda())
+        if ragged:
+            rng = np.random.Generator(np.random.PCG64(60 + i))
+            Leff = rng.integers(0, L + 1, B).astype(np.int32)
+            Leff[:2] = [0, L]
+            s["L_eff"] = torch.from_numpy(Leff).cuda()
+            s["mu_target_bonus"] = torch.from_numpy(rng.standard_normal((B, d)).astype(np.float32)).cuda().to(s["x"].dtype)
+            s["sigma_bonus"] = torch.from_numpy(rng.uniform(0.1, 1.0, B).astype(np.float32)).cuda()
+        out.append(s)
+    return out
+
+
+def _call(api, s, seed, mode, ws, out=None, pipelined=False):
+    kw = {k: s[k] for k in ("L_eff", "mu_target_bonus", "sigma_bonus") if k in s}
+    return api.verify(s["x"], s["mq"], s["mp"], s["sigma"], seed, mode, with_aux=True, workspace=ws,
+                      out=out, pipelined=pipelined, **kw)
+
+
+def _same(a, b, mask=None):
+    for k in KEYS:
+        x, y = a[k], b[k]
+        if mask is not None and k in ("y", "aux", "status"):
+            x, y = x[mask], y[mask]
+        assert torch.equal(x.view(torch.int16) if x.dtype == torch.bfloat16 else x,
+                           y.view(torch.int16) if y.dtype == torch.bfloat16 else y) or \
+            torch.equal(torch.nan_to_num(x.float(), nan=1234.5), torch.nan_to_num(y.float(), nan=1234.5)), k
+
+
+CASES = [("pixel", 64, 8, 3072, False), ("latent", 16, 16, 16384, False), ("pixel", 40, 6, 1000, True),
+         ("tiny", 8, 4, 37, True)]
+
+
+@pytest.mark.parametrize("kind,B,L,d,ragged", CASES)
+@pytest.mark.parametrize("mode", ["block", "sample"])
+def test_pipelined_calls_equal_plain_calls(api, kind, B, L, d, ragged, mode):
+    sets = _sets(kind, 4, B, L, d, ragged)
+    dt = sets[0]["x"].dtype
+    ws = torch.zeros(api.workspace_bytes(B, L, d, dt), dtype=torch.uint8, device="cuda")
+    n = 12
+    torch.cuda.synchronize()
+    piped = [_call(api, sets[i % 4], 100 + i, mode, ws, pipelined=True) for i in range(n)]
+    torch.cuda.synchronize()
+    for i in range(n):
+        ref = _call(api, sets[i % 4], 100 + i, mode, ws)
+        act = torch.ones(B, dtype=torch.bool, device="cuda") if not ragged else sets[i % 4]["L_eff"] > 0
+        _same(piped[i], ref, act)
+
+
+@pytest.mark.parametrize("kind,B,L,d,ragged", CASES[:2])
+def test_pipelined_calls_sharing_outputs(api, kind, B, L, d, ragged):
+    """Every call writes the same output buffers; they end with the last call's outputs."""
+    sets = _sets(kind, 3, B, L, d, ragged)
+    dt = sets[0]["x"].dtype
+    ws = torch.zeros(api.workspace_bytes(B, L, d, dt), dtype=torch.uint8, device="cuda")
+    out = {}
+    first = _call(api, sets[0], 7, "block", ws, out=out, pipelined=True)
+    out.update(first)
+    for i in range(1, 10):
+        r = _call(api, sets[i % 3], 7 + i, "block", ws, out=out, pipelined=True)
+    torch.cuda.synchronize()
+    ref = _call(api, sets[9 % 3], 16, "block", ws)
+    _same(r, ref)
+
+
+def test_pipelined_calls_in_a_cuda_graph(api):
+    kind, B, L, d = "pixel", 96, 8, 3072
+    sets = _sets(kind, 4, B, L, d, False)
+    ws = torch.zeros(api.workspace_bytes(B, L, d, torch.float32), dtype=torch.uint8, device="cuda")
+    outs = [dict(accepted_len=torch.empty(B, dtype=torch.int32, device="cuda"),
+                 y=torch.empty(B, d, device="cuda"), status=torch.empty(B, dtype=torch.int32, device="cuda"),
+                 log_ratio=torch.empty(B, L, device="cuda"), delta_norm=torch.empty(B, L, device="cuda"),
+                 aux=torch.empty(B, 4, device="cuda")) for _ in range(8)]
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        _call(api, sets[0], 1, "block", ws)          # warm-up outside capture
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(8):
+            _call(api, sets[i % 4], 300 + i, "block", ws, out=outs[i], pipelined=True)
+    for _ in range(2):
+        for o in outs:
+            for v in o.values():
+                v.fill_(-7)
+        g.replay()
+        torch.cuda.synchronize()
+        for i in range(8):
+            _same(outs[i], _call(api, sets[i % 4], 300 + i, "block", ws))

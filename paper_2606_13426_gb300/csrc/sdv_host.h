@@ -33,13 +33,14 @@ constexpr int64_t kK4MinChunk = 1024;
 constexpr int64_t kK4MaxChunk = 4096;
 constexpr int64_t kK4TargetCtas = 1024;
 // Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
-// finishes the chain inside the fused kernel (the residual's noise cached in dynamic
-// shared memory: up to 64 KB, 3 resident CTAs per SM), kFinishMaxGroups on the
-// many-chain path (a static 16 KB cache in k_finish); longer rows by
-// k_resid_dot/_write.  The fused kernel's residual sweeps take kFusedResidUnroll
-// groups per thread, their loads issued together.
-constexpr int64_t kFusedMaxGroups = 4096;
+// finishes the chain inside the fused kernel, kFinishMaxGroups by k_finish on the
+// many-chain path, and kPipeMaxGroups by k_finish on the pipelined path (in each case
+// the residual's noise cached in dynamic shared memory: 16 KB, or up to 64 KB);
+// longer rows by k_resid_dot/_write.  The fused kernel's residual sweeps take
+// kFusedResidUnroll groups per thread, their loads issued together.
+constexpr int64_t kFusedMaxGroups = 1024;
 constexpr int64_t kFinishMaxGroups = 1024;
+constexpr int64_t kPipeMaxGroups = 4096;
 constexpr int kFusedResidUnroll = 3;
 
 enum : int32_t {

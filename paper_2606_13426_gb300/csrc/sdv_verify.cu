@@ -798,27 +798,68 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   const int c = (int)(tile - r * C);
   const int b = (int)(r / L), j = (int)(r - (int64_t)b * L);
   const int g = A.S.L_eff ? max(0, min(A.S.L_eff[b], L)) : L;
-  if (j >= g) return;  // CTA-uniform
-  const int64_t e0 = (int64_t)c * A.chunk;
-  const int64_t e1 = min(e0 + A.chunk, A.d);
-  const float2 s = tile_sums<T, VEC, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
-  const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
-  if (threadIdx.x == 0) A.part[tile] = t;
+  if (j < g) {  // CTA-uniform
+    const int64_t e0 = (int64_t)c * A.chunk;
+    const int64_t e1 = min(e0 + A.chunk, A.d);
+    const float2 s = tile_sums<T, VEC, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
+    const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
+    if (threadIdx.x == 0) {
+      A.part[tile] = t;
+      // release the partial; k_finish acquires every partial of the chain with the count
+      ticket_acq_rel(A.ticket + b);
+    }
+  }
+  if (blockIdx.x == 0) {
+    // CTA 0 ties this grid's completion to the previous kernel's (so the next k_finish,
+    // which writes its outputs after this grid has completed, writes after the previous
+    // call's k_finish); it triggers first, its own tile done, so that k_finish can start
+    __syncthreads();
+    griddep_launch_dependents();
+    if (threadIdx.x == 0) griddep_wait();
+  }
 }
 
-// One CTA per chain: warp 0 scans the chain and draws U (warp U-sampler) while the
-// other warps draw the residual's G into shared memory; then, with RESID = 1, all
-// kFinishThreads threads write y (launched with 32 threads and leaving the chain
-// state for k_resid_* when RESID = 0).
+// One CTA per chain: warp 0 reads the chain's partials (after acquiring its tile count,
+// complete because k_finish starts only after every k_tiles CTA has taken its ticket and
+// exited or triggered), resets the count, and the CTA triggers its dependents; then warp 0 scans the chain and draws U
+// (warp U-sampler) while the other warps draw the residual's G into shared memory
+// (dynamic, (d + 3)/4 float4), and, with RESID = 1, all kFinishThreads threads write y
+// (launched with 32 threads and leaving the chain state for k_resid_* when RESID = 0).
+// Every output is written after griddep_wait.
 template <typename T, bool VEC4, int RESID>
 __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
   __shared__ ChainState cs_s;
   __shared__ float2 red[kFinishThreads / 32];
   __shared__ float bcast;
-  __shared__ float4 g_s[RESID ? kFinishMaxGroups : 1];  // the residual's G, drawn once
+  __shared__ float ell_s[SDV_MAX_L], dn_s[SDV_MAX_L];
+  extern __shared__ float4 g_s[];  // RESID: the residual's G, drawn once
   const int b = blockIdx.x;
+  const int L = A.S.L;
+  ScanRegs R;
   if (threadIdx.x < 32) {
-    const ScanOut so = scan_warp(A.S, b);
+    const int g = A.S.L_eff ? max(0, min(A.S.L_eff[b], L)) : L;
+    uint32_t cnt = 0u;
+    if (threadIdx.x == 0) {
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(cnt) : "l"(A.ticket + b) : "memory");
+      A.ticket[b] = 0u;
+    }
+    __syncwarp();
+    R = scan_load(A.S, b);
+    if (threadIdx.x == 0 && cnt != (uint32_t)(g * A.S.C)) R.any_bad = true;  // a count that cannot occur
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      if (threadIdx.x + 32 * q < L) {
+        ell_s[threadIdx.x + 32 * q] = R.ell[q];
+        dn_s[threadIdx.x + 32 * q] = R.dn[q];
+      }
+    }
+    __threadfence();
+  }
+  __syncthreads();
+  griddep_launch_dependents();  // this chain's partials are read and its count is reset
+  if (threadIdx.x < 32) {
+    R.any_bad = __any_sync(0xffffffffu, R.any_bad);
+    const ScanOut so = scan_decide(A.S, b, R);
     ChainState cs = so.cs;
     if (cs.kind == kKindResid && A.S.draw_u) {
       const uint32_t wbits = philox_block(seed_of(A.S), (uint32_t)b, 0u, kStreamUSample, 0u).x;
@@ -827,20 +868,32 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
       cs.U = usample_warp(Q, wbits, &st);
       cs.status = st;
     }
-    report_chain(A.S, b, cs, threadIdx.x == 0);
-    if (threadIdx.x == 0) {
-      if (RESID == 0) A.state[b] = cs;
-      else cs_s = cs;
-    }
+    if (threadIdx.x == 0) cs_s = cs;
   } else if (RESID) {
     prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, kFinishThreads - 32, g_s);
   }
-  if (RESID == 0) return;
   __syncthreads();
   const ChainState cs = cs_s;
-  residual_row<T, VEC4, kFinishResidUnroll, 2>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
-                                            (const T*)A.mq_bonus, A.sigma_bonus, A.S.L, A.d, seed_of(A.S),
-                                            b, cs, (T*)A.y, CtaGroup{red, &bcast}, g_s);
+  const CtaGroup grp{red, &bcast};
+  float coef = 0.f;
+  if (RESID)
+    coef = residual_coef<T, VEC4, kFinishResidUnroll, 2>((const T*)A.mq, (const T*)A.mp, L, A.d, seed_of(A.S), b,
+                                                         cs, grp, g_s);
+  // outputs: after k_tiles has completed, and with it the previous call (see k_tiles)
+  griddep_wait();
+  for (int i = threadIdx.x; i < L; i += blockDim.x) {
+    if (A.S.ell_out) A.S.ell_out[(int64_t)b * L + i] = ell_s[i];
+    if (A.S.dn_out) A.S.dn_out[(int64_t)b * L + i] = dn_s[i];
+  }
+  if (threadIdx.x == 0) {
+    scan_write_chain(A.S, b, cs);
+    report_chain(A.S, b, cs, true);
+    if (RESID == 0) A.state[b] = cs;
+  }
+  if (RESID)
+    residual_write<T, VEC4, kFinishResidUnroll, 2>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
+                                                   (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S), b,
+                                                   cs, coef, (T*)A.y, grp, g_s);
 }
 
 // ---------------------------------------------------------------- acceptance scan only
@@ -1072,19 +1125,18 @@ static int validate_window(const void* x, const void* mq, const void* mp, const 
   return SDV_OK;
 }
 
-// One launch of k_verify: dynamic shared memory for the residual's noise cache (RESID),
-// and, with `overlap`, the programmatic-serialisation attribute that lets the kernel
-// start before the previous kernel on the stream has finished.
+// A launch through cudaLaunchKernelEx: dynamic shared memory (raising the kernel's limit
+// when it passes 48 KB) and, with `overlap`, programmatic stream serialisation.
 template <typename Kern>
-static cudaError_t launch_k1(Kern kern, unsigned tiles, size_t smem, bool overlap, const VerifyArgs& A,
-                             cudaStream_t s) {
+static cudaError_t launch_ex(Kern kern, unsigned grid, unsigned threads, size_t smem, bool overlap,
+                             const VerifyArgs& A, cudaStream_t s) {
   if (smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(tiles);
-  cfg.blockDim = dim3(kK1Threads);
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute at[1];
@@ -1105,7 +1157,7 @@ static cudaError_t launch_verify(const VerifyArgs& A, int B, int L, int vpt, boo
                     (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
   const unsigned tiles = (unsigned)((int64_t)B * L * A.S.C);
   const size_t smem = (RESID && !A.S.ratios_only) ? sizeof(float4) * (size_t)((A.d + 3) / 4) : 0;
-#define SDV_LAUNCH(VECV, VPTV, V4) return launch_k1(k_verify<T, VECV, VPTV, V4, RESID, RU>, tiles, smem, overlap, A, s)
+#define SDV_LAUNCH(VECV, VPTV, V4) return launch_ex(k_verify<T, VECV, VPTV, V4, RESID, RU>, tiles, kK1Threads, smem, overlap, A, s)
   if (!vec) {
     if (vec4) SDV_LAUNCH(false, 1, true);
     SDV_LAUNCH(false, 1, false);
@@ -1128,30 +1180,28 @@ static cudaError_t launch_verify(const VerifyArgs& A, int B, int L, int vpt, boo
 }
 
 template <typename T>
-static void launch_tiles(const VerifyArgs& A, int B, int L, int vpt, cudaStream_t s) {
+static cudaError_t launch_tiles(const VerifyArgs& A, int B, int L, int vpt, bool overlap, cudaStream_t s) {
   constexpr int V = 16 / (int)sizeof(T);
   const bool vec = (A.d % V == 0) && aligned(A.x, 16) && aligned(A.mq, 16) && aligned(A.mp, 16);
   const unsigned tiles = (unsigned)((int64_t)B * L * A.S.C);
-  if (!vec) {
-    k_tiles<T, false, 1><<<tiles, kK1Threads, 0, s>>>(A);
-    return;
-  }
+  if (!vec) return launch_ex(k_tiles<T, false, 1>, tiles, kK1Threads, 0, overlap, A, s);
   switch (vpt) {
-    case 1: k_tiles<T, true, 1><<<tiles, kK1Threads, 0, s>>>(A); break;
-    case 2: k_tiles<T, true, 2><<<tiles, kK1Threads, 0, s>>>(A); break;
-    case 3: k_tiles<T, true, 3><<<tiles, kK1Threads, 0, s>>>(A); break;
-    default: k_tiles<T, true, 4><<<tiles, kK1Threads, 0, s>>>(A); break;
+    case 1: return launch_ex(k_tiles<T, true, 1>, tiles, kK1Threads, 0, overlap, A, s);
+    case 2: return launch_ex(k_tiles<T, true, 2>, tiles, kK1Threads, 0, overlap, A, s);
+    case 3: return launch_ex(k_tiles<T, true, 3>, tiles, kK1Threads, 0, overlap, A, s);
+    default: return launch_ex(k_tiles<T, true, 4>, tiles, kK1Threads, 0, overlap, A, s);
   }
 }
 
 template <typename T, int RESID>
-static void launch_finish(const VerifyArgs& A, int B, cudaStream_t s) {
+static cudaError_t launch_finish(const VerifyArgs& A, int B, bool overlap, cudaStream_t s) {
   const bool vec4 = (A.d % 4 == 0) && aligned(A.x, 4 * sizeof(T)) && aligned(A.mq, 4 * sizeof(T)) &&
                     aligned(A.mp, 4 * sizeof(T)) && (A.y == nullptr || aligned(A.y, 4 * sizeof(T))) &&
                     (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
-  const int nt = RESID ? kFinishThreads : 32;
-  if (vec4) k_finish<T, true, RESID><<<B, nt, 0, s>>>(A);
-  else k_finish<T, false, RESID><<<B, nt, 0, s>>>(A);
+  const unsigned nt = RESID ? kFinishThreads : 32;
+  const size_t smem = RESID ? sizeof(float4) * (size_t)((A.d + 3) / 4) : 0;
+  if (vec4) return launch_ex(k_finish<T, true, RESID>, (unsigned)B, nt, smem, overlap, A, s);
+  return launch_ex(k_finish<T, false, RESID>, (unsigned)B, nt, smem, overlap, A, s);
 }
 
 template <typename T>
@@ -1202,31 +1252,32 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
 
   cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
-  const bool many = !ratios_only && B >= kManyChainMin;
-  // rows whose residual the finishing CTA writes itself (k_verify: its noise cache in
-  // dynamic shared memory; k_finish: a static cache); longer rows go to k_resid_*
-  const bool long_rows = !ratios_only && (d + 3) / 4 > (many ? kFinishMaxGroups : kFusedMaxGroups);
+  const int64_t ng = (d + 3) / 4;
+  // Paths: a pipelined call whose rows fit the finishing CTA's noise cache streams with
+  // k_tiles and finishes with k_finish, both launched to overlap their predecessors;
+  // otherwise the fused kernel (fewer than kManyChainMin chains) or k_tiles + k_finish
+  // (many chains), with the residual of rows longer than the finishing CTA's cache left to
+  // k_resid_dot / k_resid_write.
+  overlap = overlap && !ratios_only && ng <= kPipeMaxGroups;
+  const bool many = !ratios_only && (overlap || B >= kManyChainMin);
+  const bool long_rows = !ratios_only && !overlap && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
-  // consecutive calls may overlap only on the single-kernel path
-  overlap = overlap && !many && !long_rows;
   cudaError_t e = cudaSuccess;
+  // the tickets return to zero at the end of every call; a pipelined call relies on
+  // that (the caller's contract), the others clear them first
+  if (!overlap && cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+    check_launch();
+    return SDV_ECUDA;
+  }
   if (many) {
-    if (f32) launch_tiles<float>(A, B, L, w.vpt1, s);
-    else launch_tiles<__nv_bfloat16>(A, B, L, w.vpt1, s);
+    e = f32 ? launch_tiles<float>(A, B, L, w.vpt1, overlap, s)
+            : launch_tiles<__nv_bfloat16>(A, B, L, w.vpt1, overlap, s);
+  } else if (long_rows) {
+    e = f32 ? launch_verify<float, 0>(A, B, L, w.vpt1, false, s)
+            : launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, false, s);
   } else {
-    // the tickets return to zero at the end of every call; a call that may overlap
-    // its predecessor relies on that (the caller's contract), the others clear them
-    if (!overlap && cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
-      check_launch();
-      return SDV_ECUDA;
-    }
-    if (long_rows) {
-      e = f32 ? launch_verify<float, 0>(A, B, L, w.vpt1, false, s)
-              : launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, false, s);
-    } else {
-      e = f32 ? launch_verify<float, 1>(A, B, L, w.vpt1, overlap, s)
-              : launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, overlap, s);
-    }
+    e = f32 ? launch_verify<float, 1>(A, B, L, w.vpt1, false, s)
+            : launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, false, s);
   }
   if (e != cudaSuccess) {
     g_last_cuda_error = (int)e;
@@ -1237,12 +1288,14 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   if (rc != SDV_OK) return rc;
   if (tev) timing_record(tev[1], s);
   if (many) {
-    if (long_rows) {
-      if (f32) launch_finish<float, 0>(A, B, s);
-      else launch_finish<__nv_bfloat16, 0>(A, B, s);
-    } else {
-      if (f32) launch_finish<float, 1>(A, B, s);
-      else launch_finish<__nv_bfloat16, 1>(A, B, s);
+    if (long_rows)
+      e = f32 ? launch_finish<float, 0>(A, B, overlap, s) : launch_finish<__nv_bfloat16, 0>(A, B, overlap, s);
+    else
+      e = f32 ? launch_finish<float, 1>(A, B, overlap, s) : launch_finish<__nv_bfloat16, 1>(A, B, overlap, s);
+    if (e != cudaSuccess) {
+      g_last_cuda_error = (int)e;
+      cudaGetLastError();
+      return SDV_ECUDA;
     }
     if ((rc = check_launch()) != SDV_OK) return rc;
   }

@@ -7,7 +7,8 @@ Tolerances (from the verification step's accuracy targets):
     within the tie band of its threshold: |log eta_j - log thr_j| < 1e-4 plus the
     propagated log-ratio tolerance (thr = min{1, e^ell} in sample mode, h_j in block
     mode, where log alpha_j accumulates the tolerance of ell_1..ell_j);
-  * output states (chains with equal tau): 1e-5 absolute for fp32 inputs, 2e-2 for bf16.
+  * output states (chains with equal tau): 1e-5 absolute for fp32 inputs, 2e-2 for bf16
+    (widened to half a bf16 ulp where |y| > 5.12; y_tolerance).
 """
 import numpy as np
 import torch
@@ -16,6 +17,16 @@ from oracle import philox as OP
 from oracle import verify as OV
 
 TOL_Y = {"f32": 1e-5, "bf16": 2e-2}
+
+
+def y_tolerance(y_ref, dtype):
+    """Output-state tolerance: 1e-5 absolute for fp32; 2e-2 absolute for bf16, widened
+    to the output's own rounding, half a bf16 ulp (at most 2^-8 |y|), where |y| > 5.12:
+    a bf16 state of magnitude 8 or more is 0.0625 from its neighbours, so no
+    implementation that stores y in bf16 can be within 2e-2 of every value there."""
+    if dtype == "bf16":
+        return np.maximum(TOL_Y["bf16"], 2.0 ** -8 * np.abs(y_ref))
+    return TOL_Y[dtype]
 
 
 def to_dev(inp, name):
@@ -119,8 +130,9 @@ def compare(g, o, mode, dtype, omega=1.0, max_tie_frac=0.05):
     yg, yo = g["y"][same], o["y"][same]
     act = np.isfinite(yo).all(axis=1)          # inactive chains emit nothing
     err = np.abs(yg[act] - yo[act])
-    tol = TOL_Y[dtype]
-    assert err.size == 0 or err.max() <= tol, "y max err %g (tol %g)" % (err.max(), tol)
+    tol = y_tolerance(yo[act], dtype)
+    assert err.size == 0 or np.all(err <= tol), "y max err %g (tol %g)" % (
+        err.max(), tol if np.isscalar(tol) else tol.flat[np.argmax(err)])
     assert np.array_equal(g["status"][same][act] & 3, o["status"][same][act] & 3)
     return int(diff.sum())
 

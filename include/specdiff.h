@@ -156,8 +156,10 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  * call may start streaming its window before the previous kernel on `stream` has
  * finished, so that the latency-bound end of one call (the last chains' acceptance
  * rule, U-draw and residual) overlaps the next call's read of its window.  The
- * verification itself is the same (Algorithms block-verification, decomposition-res,
- * u-sample); the results equal sdv_verify_ex's for the same arguments.
+ * verification itself is the same (Algorithms token-/block-verification,
+ * decomposition-res, u-sample): log ratios, accepted lengths and status equal
+ * sdv_verify_ex's bit for bit; U and y agree within the library's accuracy (rows of
+ * up to 4096 elements finish in a 64-thread CTA with the one-warp U-sampler).
  * Preconditions (the caller's promise; nothing checks them):
  *   - the window (x_draft, mu_target, mu_draft, sigma, L_eff, mu_target_bonus,
  *     sigma_bonus) is not written by earlier work on `stream` that may still be
@@ -166,11 +168,11 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  *   - the workspace's counters are zero: the workspace is fresh from a
  *     cudaMemset to 0, or was last used by a completed call of this library
  *     (every call leaves them at zero).
- * Outputs are written only after the previous kernel on `stream` has completed,
- * so consecutive calls may share output buffers.  The overlap applies where a call
- * is one kernel (B < 512 chains and rows of at most 16384 elements); other calls
- * run exactly as sdv_verify_ex.  Same arguments, return codes and ownership as
- * sdv_verify_ex; the workspace must not be shared with calls on other streams.
+ * Outputs are written only after the previous call on `stream` has written its own,
+ * so consecutive calls may share output buffers.  The overlap applies to rows of up
+ * to 16384 elements; longer rows run exactly as sdv_verify_ex.  Same arguments,
+ * return codes and ownership as sdv_verify_ex; the workspace must not be shared with
+ * calls on other streams.
  */
 int sdv_verify_pipelined(const void *x_draft, const void *mu_target, const void *mu_draft,
                          const float *sigma, int64_t sigma_stride_b,

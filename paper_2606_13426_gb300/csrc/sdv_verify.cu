@@ -805,8 +805,9 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
     const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
     if (threadIdx.x == 0) {
       A.part[tile] = t;
-      // release the partial; k_finish acquires every partial of the chain with the count
-      ticket_acq_rel(A.ticket + b);
+      // release the partial with the chain's count, which wraps to 0 at the chain's
+      // last tile; k_finish acquires every partial of the chain by reading that 0
+      ticket_inc(A.ticket + b, (unsigned int)(g * C) - 1u);
     }
   }
   if (blockIdx.x == 0) {
@@ -820,8 +821,8 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
 }
 
 // One CTA per chain: warp 0 reads the chain's partials (after acquiring its tile count,
-// complete because k_finish starts only after every k_tiles CTA has taken its ticket and
-// exited or triggered), resets the count, and the CTA triggers its dependents; then warp 0 scans the chain and draws U
+// complete -- and wrapped back to 0 -- because k_finish starts only after every k_tiles
+// CTA has taken its ticket and exited or triggered), and the CTA triggers its dependents; then warp 0 scans the chain and draws U
 // (warp U-sampler) while the other warps draw the residual's G into shared memory
 // (dynamic, (d + 3)/4 float4), and, with RESID = 1, all kFinishThreads threads write y
 // (launched with 32 threads and leaving the chain state for k_resid_* when RESID = 0).
@@ -837,15 +838,15 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
   const int L = A.S.L;
   ScanRegs R;
   if (threadIdx.x < 32) {
-    const int g = A.S.L_eff ? max(0, min(A.S.L_eff[b], L)) : L;
-    uint32_t cnt = 0u;
     if (threadIdx.x == 0) {
+      // the count is back at 0 after the chain's last tile: reading it with acquire
+      // semantics makes every partial released by the chain's tiles visible
+      uint32_t cnt;
       asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(cnt) : "l"(A.ticket + b) : "memory");
-      A.ticket[b] = 0u;
+      (void)cnt;
     }
     __syncwarp();
     R = scan_load(A.S, b);
-    if (threadIdx.x == 0 && cnt != (uint32_t)(g * A.S.C)) R.any_bad = true;  // a count that cannot occur
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
       if (threadIdx.x + 32 * q < L) {
@@ -853,12 +854,10 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
         dn_s[threadIdx.x + 32 * q] = R.dn[q];
       }
     }
-    __threadfence();
   }
   __syncthreads();
-  griddep_launch_dependents();  // this chain's partials are read and its count is reset
+  griddep_launch_dependents();  // this chain's partials are read
   if (threadIdx.x < 32) {
-    R.any_bad = __any_sync(0xffffffffu, R.any_bad);
     const ScanOut so = scan_decide(A.S, b, R);
     ChainState cs = so.cs;
     if (cs.kind == kKindResid && A.S.draw_u) {
@@ -1253,13 +1252,16 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
   const int64_t ng = (d + 3) / 4;
-  // Paths: a pipelined call whose rows fit the finishing CTA's noise cache streams with
-  // k_tiles and finishes with k_finish, both launched to overlap their predecessors;
-  // otherwise the fused kernel (fewer than kManyChainMin chains) or k_tiles + k_finish
-  // (many chains), with the residual of rows longer than the finishing CTA's cache left to
-  // k_resid_dot / k_resid_write.
+  // Paths.  A pipelined call (overlap) with rows of up to kFinishMaxGroups groups of four
+  // streams with k_tiles and finishes with k_finish, both launched to overlap their
+  // predecessors; with rows of up to kPipeMaxGroups it runs the fused kernel, launched
+  // to overlap its predecessor, with the residual's noise cache in up to 64 KB of
+  // dynamic shared memory (k_finish's 64 threads would write such rows too slowly).
+  // Otherwise the fused kernel (fewer than kManyChainMin chains) or k_tiles + k_finish
+  // (many chains), with the residual of rows longer than the finishing CTA's cache left
+  // to k_resid_dot / k_resid_write.
   overlap = overlap && !ratios_only && ng <= kPipeMaxGroups;
-  const bool many = !ratios_only && (overlap || B >= kManyChainMin);
+  const bool many = !ratios_only && (overlap ? ng <= kFinishMaxGroups : B >= kManyChainMin);
   const bool long_rows = !ratios_only && !overlap && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;
@@ -1276,8 +1278,8 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
     e = f32 ? launch_verify<float, 0>(A, B, L, w.vpt1, false, s)
             : launch_verify<__nv_bfloat16, 0>(A, B, L, w.vpt1, false, s);
   } else {
-    e = f32 ? launch_verify<float, 1>(A, B, L, w.vpt1, false, s)
-            : launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, false, s);
+    e = f32 ? launch_verify<float, 1>(A, B, L, w.vpt1, overlap, s)
+            : launch_verify<__nv_bfloat16, 1>(A, B, L, w.vpt1, overlap, s);
   }
   if (e != cudaSuccess) {
     g_last_cuda_error = (int)e;

@@ -269,6 +269,17 @@ int sdv_philox(const uint32_t *ctr, uint64_t seed, int n, uint32_t *out, sdv_str
 int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub,
                 float *out, sdv_stream_t stream);
 
+/*
+ * sdv_special - the special functions the acceptance rule and the U-sampler build on,
+ * evaluated by the kernels' own device code at n points z (fp32 device arrays):
+ *   which = 0: erfcx(z) = exp(z^2) erfc(z) (the library's own approximation)
+ *   which = 1: log Phi(z)
+ *   which = 2: g'(z) = lambda(z) + z, lambda = phi/Phi (inverse Mills ratio)
+ * (App. "Density ratio calculations": the CDF differences of h_j and Eq. u-cdf are
+ * evaluated from these in log space.)  out[i] for z[i]; SDV_EINVAL for another which.
+ */
+int sdv_special(int which, const float *z, int n, float *out, sdv_stream_t stream);
+
 /* ---- end-to-end sampler on an analytic Gaussian-mixture target --------------
  *
  * Model (Eq. forward-process, backward-process, target-distribution): a

@@ -247,6 +247,13 @@ def normals(seed, Bn, d, stream_id, sub=0, device="cuda"):
     return out
 
 
+def special(which, z):
+    """The device special functions (sdv_special): 'erfcx', 'log_ndtr' or 'gprime' at z (fp32)."""
+    _need_cuda(z)
+    out = torch.empty_like(z)
+    B.sdv_special({"erfcx": 0, "log_ndtr": 1, "gprime": 2}[which], _ptr(z), z.numel(), _ptr(out), _stream())
+    return out
+
 
 class GmmTarget:
     """Analytic Gaussian-mixture target and its variance-preserving schedule (device copies)."""

@@ -61,6 +61,7 @@ SIGNATURES = {
     "sdv_usample": (_I, [_P, _P, _P, _I, _P, _P, _P]),
     "sdv_philox": (_I, [_P, _U64, _I, _P, _P]),
     "sdv_normals": (_I, [_U64, _I, _I64, _I, _U32, _P, _P]),
+    "sdv_special": (_I, [_I, _P, _I, _P, _P]),
     "sdv_gmm_target": (_I, [_P, _P, _I, _I64, _P, _P, _I, _F, _I, _F, _F, _F, _F, _P, _P, _P]),
     "sdv_free_draft": (_I, [_P, _P, _P, _P, _I, _I, _I64, _I, _F, _F, _F, _F, _U64, _P, _P, _P,
                             _P]),
@@ -194,6 +195,10 @@ def sdv_philox(ctr, seed, n, out, stream):
 
 def sdv_normals(seed, B, d, stream_id, sub, out, stream):
     return _call("sdv_normals", seed, B, d, stream_id, sub, out, stream)
+
+
+def sdv_special(which, z, n, out, stream):
+    return _call("sdv_special", which, z, n, out, stream)
 
 
 def sdv_timing_enable(slots):

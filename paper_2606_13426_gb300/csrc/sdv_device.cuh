@@ -127,21 +127,64 @@ constexpr float kSqrtHalf = 0.70710678118654752f;
 constexpr float kHalfLog2Pi = 0.91893853320467274f;  // log(2 pi) / 2
 constexpr float kLn2 = 0.69314718055994531f;
 
+// Reciprocal without the IEEE slow path: the hardware approximation refined by one
+// Newton step (about 1 ulp for finite non-zero x; +-inf gives 0 and 0 gives inf).
+// IEEE division and __frcp_rn branch to a slow path, which keeps independent
+// evaluations from overlapping; this form does not.
+__device__ __forceinline__ float frcp_fast(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  const float e = fmaf(-x, r, 1.0f);
+  return (r != 0.0f && isfinite(r)) ? fmaf(r, e, r) : r;
+}
+
 // 8-point Gauss-Legendre nodes / weights on [-1, 1] (positive half).
 static __constant__ float kGLx[4] = {0.18343464249564978f, 0.52553240991632899f,
                                           0.79666647741362673f, 0.96028985649753618f};
 static __constant__ float kGLw[4] = {0.36268378337836166f, 0.31370664587788688f,
                                           0.22238103445337443f, 0.10122853629037706f};
 
-// One shared copy of the scaled complementary error function (see SDV_GL_UNROLL).
-static __device__ SDV_HELPER float erfcx_f(float x) { return erfcxf(x); }
+// The scaled complementary error function erfcx(z) = exp(z^2) erfc(z), branch-free and
+// inline so that independent evaluations (the quadrature nodes below) overlap.  For
+// z >= 0: erfcx(z) = t exp(f(t)), t = 1/(1 + z/2), with f(t) = log(erfcx(z)/t) a
+// degree-11 polynomial in x = 2t - 1 (a Chebyshev fit of f, generated by
+// gen_erfcx_coeffs.py; max relative error 1.4e-7 in fp32).  z = +inf gives t = 0 and 0.
+__device__ __forceinline__ float erfcx_pos(float z) {
+  const float t = frcp_fast(fmaf(0.5f, z, 1.0f));
+  const float x = fmaf(2.0f, t, -1.0f);
+  // f(t) = log(erfcx(z)/t) in the power basis of x = 2t - 1, degree 11 (Horner)
+  float f = -8.728381024e-05f;
+  f = fmaf(f, x, 8.000738166e-06f);
+  f = fmaf(f, x, 5.737663720e-04f);
+  f = fmaf(f, x, -2.279109660e-04f);
+  f = fmaf(f, x, -2.288765239e-03f);
+  f = fmaf(f, x, 1.794066250e-03f);
+  f = fmaf(f, x, 8.808825369e-03f);
+  f = fmaf(f, x, -9.880019324e-03f);
+  f = fmaf(f, x, -4.689364056e-02f);
+  f = fmaf(f, x, 4.734388761e-02f);
+  f = fmaf(f, x, 6.726431548e-01f);
+  f = fmaf(f, x, -6.717940917e-01f);
+  return t * expf(f);
+}
+
+// erfcx of any sign: erfcx(-a) = 2 exp(a^2) - erfcx(a) (no cancellation: the first
+// term is at least 2, the second at most 1), with a^2 split exactly (hi + lo) so that
+// exp(a^2) keeps full relative accuracy; overflows to +inf for a above ~9.4.
+__device__ __forceinline__ float erfcx_any(float z) {
+  const float a = fabsf(z);
+  const float e = erfcx_pos(a);
+  const float hi = a * a, lo = fmaf(a, a, -hi);
+  const float big = 2.0f * expf(hi) * (1.0f + lo);
+  return (z >= 0.0f) ? e : big - e;
+}
 
 // (log Phi(a), g(a)) from one scaled complement E = erfcx(|a|/sqrt 2)/2 =
 // Phi(-|a|) e^{a^2/2}: for a <= 0, log Phi(a) = log E - a^2/2 (no underflow); for
 // a > 0, log Phi(a) = log(1 - E e^{-a^2/2}).  Both branches are computed and one is
 // selected, so that lanes with different arguments do not diverge.
 __device__ __forceinline__ float2 log_ndtr_g(float a) {
-  const float E = 0.5f * erfcx_f(fabsf(a) * kSqrtHalf);
+  const float E = 0.5f * erfcx_pos(fabsf(a) * kSqrtHalf);
   const float h = 0.5f * a * a;
   const float lneg = logf(E);                  // log Phi(-|a|) + a^2/2
   const float lpos = log1pf(-E * expf(-h));    // log Phi(|a|)
@@ -163,7 +206,7 @@ static __device__ SDV_HELPER float gfun(float a) { return log_ndtr_g(a).y; }
 // sqrt(2/pi)/erfcx(-s/sqrt 2) + s, which tends to s for large s as erfcx overflows.
 __device__ __forceinline__ float gprime_cf(float s) {
   const float x = fmaxf(-s, 4.0f);
-  const float u = 1.0f / (x * x);
+  const float u = frcp_fast(x * x);
   float a0 = 1.0f, a1 = 1.0f, b0 = 0.0f, b1 = 1.0f;  // A_{n-2}, A_{n-1}, B_{n-2}, B_{n-1}
 #pragma unroll
   for (int n = 2; n <= 16; ++n) {
@@ -171,10 +214,12 @@ __device__ __forceinline__ float gprime_cf(float s) {
     const float a2 = fmaf(an, a0, a1), b2 = fmaf(an, b0, b1);
     a0 = a1; a1 = a2; b0 = b1; b1 = b2;
   }
-  return b1 / (x * a1);
+  return b1 * frcp_fast(x * a1);
 }
 __device__ __forceinline__ float gprime_ex(float s) {
-  return 0.79788456080286536f / erfcx_f(-s * kSqrtHalf) + s;
+  // lambda(s) = sqrt(2/pi) / erfcx(-s/sqrt 2); erfcx = +inf (s above ~13) gives 0
+  const float e = erfcx_any(-s * kSqrtHalf);
+  return (isinf(e) ? 0.0f : __fdividef(0.79788456080286536f, e)) + s;
 }
 
 // g(hi) - g(hi - h) for h >= 0; the interval length is exactly h.  The direct
@@ -271,7 +316,7 @@ __device__ __forceinline__ float block_log_h(float la, float Dn, float lv) {
 static __device__ SDV_HELPER float block_log_h(float la, float Dn) {
   if (isnan(la) || isnan(Dn) || !(la < 0.0f) || la == -INFINITY || !(Dn > 0.0f))
     return block_log_h(la, Dn, 0.0f);  // the limits, which do not read log v
-  const float ap = la / Dn + 0.5f * Dn;
+  const float ap = la * frcp_fast(Dn) + 0.5f * Dn;
   const float x0 = -gdiff(ap, Dn);              // log(Phi(a-) / (alpha Phi(a+)))
   const float lv = la + log_ndtr(ap) + log1mexp(x0);
   return block_log_h(la, Dn, lv);
@@ -291,7 +336,7 @@ static __device__ SDV_HELPER UParams usample_setup(float D, float la) {
   UParams P;
   P.D = D;
   P.la = la;
-  P.ap = la / D + 0.5f * D;
+  P.ap = la * frcp_fast(D) + 0.5f * D;
   P.am = P.ap - D;
   const float x0 = -gdiff(P.ap, D);
   const float2 lg = log_ndtr_g(P.ap);
@@ -365,7 +410,7 @@ __device__ __forceinline__ float usample_newton(const UParams& P, bool upper, fl
   const float lden = upper ? ge + target : target - ge;   // log(1 - Psi) or log Psi at te
   const float dg = expf(lpsi - lden);
   const float ue = P.ap - te;
-  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge / dg : 0.0f;
+  float step = (isfinite(dg) && dg > 0.0f && isfinite(ge)) ? ge * frcp_fast(dg) : 0.0f;
   step = fminf(fmaxf(step, te - hi), te - lo);   // stay inside the bracket
   return ue + step;
 }
@@ -430,7 +475,7 @@ __device__ __forceinline__ float usample_block(const UParams& P, uint32_t wbits,
     __syncthreads();
     return f;
   };
-  const float s0 = 1.0f / fmaxf(1.0f, fabsf(P.am));
+  const float s0 = frcp_fast(fmaxf(1.0f, fabsf(P.am)));
   const float tk = s0 * exp2f((float)tid * 0.125f - 8.0f);
   const float gk = gap(tk);
   int f = first_true(gk >= 0.0f);
@@ -487,7 +532,7 @@ __device__ __forceinline__ float usample_warp(const UParams& P, uint32_t wbits, 
     if (upper) return usample_log_1mpsi(t, P) - target;
     return target - usample_log_psi(t, P);
   };
-  const float s0 = 1.0f / fmaxf(1.0f, fabsf(P.am));
+  const float s0 = frcp_fast(fmaxf(1.0f, fabsf(P.am)));
   const float tk = s0 * exp2f((float)lane - 8.0f);
   const float gk = gap(tk);
   unsigned m = __ballot_sync(FULL, gk >= 0.0f);

@@ -249,8 +249,9 @@ __device__ ScanRegs scan_load(const ScanArgs& A, int b) {
         }
         const float s = A.sigma[(int64_t)b * A.sstride + j];
         R.S1[q] = a1; R.S2[q] = a2; R.sg[q] = s;
-        R.ell[q] = -(a1 + 0.5f * a2) / (s * s);
-        R.dn[q] = sqrtf(a2) / s;
+        const float rs = frcp_fast(s);
+        R.ell[q] = -(a1 + 0.5f * a2) * (rs * rs);
+        R.dn[q] = sqrtf(a2) * rs;
         if (!(s > 0.f) || !isfinite(s)) bad = true;
       } else {
         R.ell[q] = A.ell_in[(int64_t)b * L + j];
@@ -1019,6 +1020,13 @@ __global__ void k_philox(const uint4* __restrict__ ctr, uint64_t seed, int n, ui
   if (i < n) out[i] = philox4x32_10(ctr[i], (uint32_t)seed, (uint32_t)(seed >> 32));
 }
 
+__global__ void k_special(int which, const float* __restrict__ z, int n, float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float v = z[i];
+  out[i] = which == 0 ? erfcx_any(v) : (which == 1 ? log_ndtr_g(v).x : (v < -4.0f ? gprime_cf(v) : gprime_ex(v)));
+}
+
 __global__ void k_normals(uint64_t seed, int B, int64_t d, uint32_t stream, uint32_t sub, float* out) {
   const int64_t ng = (d + 3) / 4;
   const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -1469,6 +1477,14 @@ int sdv_normals(uint64_t seed, int B, int64_t d, int stream_id, uint32_t sub, fl
   if (!aligned(out, 4)) return SDV_EALIGN;
   const int64_t n = (int64_t)B * ((d + 3) / 4);
   k_normals<<<(unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream>>>(seed, B, d, (uint32_t)stream_id, sub, out);
+  return check_launch();
+}
+
+int sdv_special(int which, const float* z, int n, float* out, sdv_stream_t stream) {
+  if (!z || !out || n < 0 || which < 0 || which > 2) return SDV_EINVAL;
+  if (!aligned(z, 4) || !aligned(out, 4)) return SDV_EALIGN;
+  if (n == 0) return SDV_OK;
+  k_special<<<(n + 255) / 256, 256, 0, (cudaStream_t)stream>>>(which, z, n, out);
   return check_launch();
 }
 

@@ -335,3 +335,29 @@ def test_gpu_block_beats_sample_in_expectation(api):
         t = [run_gpu(api, inp, s, mode)["accepted_len"] + 1 for s in range(8)]
         taus[mode] = np.concatenate(t).astype(np.float64)
     assert taus["block"].mean() > taus["sample"].mean()
+
+
+# ------------------------------------------------------------------ special functions
+def test_device_special_functions(api):
+    """The kernels' own erfcx (a polynomial fit, gen_erfcx_coeffs.py), log Phi and
+    g' = lambda + z against scipy in fp64 over the ranges the acceptance rule and the
+    U-sampler reach, including the negative side of erfcx and both forms of g'."""
+    from scipy.special import erfcx, log_ndtr
+    z = np.concatenate([np.linspace(-9.0, 30.0, 20001), [0.0, 1e-8, 1e3, 1e6]]).astype(np.float32)
+    zz = torch.from_numpy(z).cuda()
+    z64 = z.astype(np.float64)
+    e = api.special("erfcx", zz).cpu().numpy().astype(np.float64)
+    ref = erfcx(z64)
+    fin = np.isfinite(ref)
+    assert np.max(np.abs(e[fin] / ref[fin] - 1.0)) < 6e-7
+    ln = api.special("log_ndtr", torch.from_numpy(np.linspace(-30, 8, 20001).astype(np.float32)).cuda())
+    x = np.linspace(-30, 8, 20001).astype(np.float32).astype(np.float64)
+    lr = log_ndtr(x)
+    err = np.abs(ln.cpu().numpy() - lr)
+    assert np.all(err <= 4e-7 * np.maximum(1.0, np.abs(lr)))
+    s = np.linspace(-60.0, 12.0, 20001).astype(np.float32)
+    gp = api.special("gprime", torch.from_numpy(s).cuda()).cpu().numpy().astype(np.float64)
+    s64 = s.astype(np.float64)
+    lam = np.exp(-0.5 * s64 * s64 - 0.5 * np.log(2 * np.pi) - log_ndtr(s64))
+    gref = lam + s64
+    assert np.all(np.abs(gp - gref) <= 1e-6 * np.maximum(1.0, np.abs(gref)) + 4e-7 * np.abs(s64))

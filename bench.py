@@ -1,8 +1,8 @@
 """Benchmark of the speculative-diffusion verification step on GB300.
 
-One step = one verification call (sdv_verify_pipelined: one fused kernel -- log-ratio
-pass, acceptance rule, residual U-draw, residual write) on one batch of the
-pixel-scale workload (B=256 chains, L=8 draft steps, d=3x32x32 fp32, block
+One step = one verification call (sdv_verify_pipelined: k_tiles streams the window and
+reduces the log-ratio partials, k_finish runs the acceptance rule, the residual U-draw
+and the residual write) on one batch of the pixel-scale workload (B=256 chains, L=8 draft steps, d=3x32x32 fp32, block
 verification) with inputs resident in HBM.  Eight input sets (8 x 75.5 MB, well
 above the 129 MB L2) rotate between steps, so every step reads its inputs from HBM.
 Steps are independent batches of chains: consecutive calls may overlap on the GPU (a
@@ -149,9 +149,11 @@ class ClockSampler:
 
 
 # Rows of more than this many groups of four elements get their residual from two
-# extra kernels (the library's kFusedMaxGroups; kFinishMaxGroups on the many-chain path).
-FUSED_MAX_GROUPS = 4096
+# extra kernels (the library's kFusedMaxGroups and kFinishMaxGroups); pipelined calls
+# keep rows of up to PIPE_MAX_GROUPS in k_finish (kPipeMaxGroups).
+FUSED_MAX_GROUPS = 1024
 FINISH_MAX_GROUPS = 1024
+PIPE_MAX_GROUPS = 4096
 
 # From this many chains on, the library streams the tiles with k_tiles and finishes
 # every chain with one warp of k_finish (the library's kManyChainMin).
@@ -162,16 +164,33 @@ def many_chains(B):
     return B >= MANY_CHAIN_MIN
 
 
-def long_rows(d, B=0):
-    """Rows whose residual two extra kernels write (longer than the fused kernel's, or on
-    the many-chain path k_finish's, noise cache)."""
+def pipelined_path(d, pipelined):
+    """Does a pipelined call of row length d take the overlapping k_tiles + k_finish path?"""
+    return pipelined and (d + 3) // 4 <= PIPE_MAX_GROUPS
+
+
+def long_rows(d, B=0, pipelined=False):
+    """Rows whose residual two extra kernels write (longer than the finishing CTA's noise
+    cache: the fused kernel's or, on the many-chain path, k_finish's)."""
+    if pipelined_path(d, pipelined):
+        return False
     return (d + 3) // 4 > (FINISH_MAX_GROUPS if many_chains(B) else FUSED_MAX_GROUPS)
 
 
-def launches_per_step(B, d):
-    """Kernels one verification call launches: the fused verify kernel (or k_tiles and
-    k_finish for many chains), plus the residual dot / write kernels for long rows."""
-    return (2 if many_chains(B) else 1) + (2 if long_rows(d, B) else 0)
+def launches_per_step(B, d, pipelined=False):
+    """Kernels one verification call launches: the fused verify kernel, or k_tiles and
+    k_finish (many chains, or a pipelined call), plus the residual dot / write kernels
+    for long rows."""
+    two = many_chains(B) or pipelined_path(d, pipelined)
+    return (2 if two else 1) + (2 if long_rows(d, B, pipelined) else 0)
+
+
+def kernels_of_step(B, d, pipelined=False):
+    two = many_chains(B) or pipelined_path(d, pipelined)
+    names = ["k_tiles", "k_finish"] if two else ["k_verify"]
+    if long_rows(d, B, pipelined):
+        names += ["k_resid_dot", "k_resid_write"]
+    return names
 
 
 def call_bytes(B, L, d, dtype):
@@ -540,10 +559,9 @@ def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clock
         roofline={"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                   "frac": achieved / hbm_peak, "peak_kind": peak_kind,
                   "kernel": ("k_verify (fused: log-ratio pass, acceptance, U-draw, residual write)"
-                             if launches_per_step(Bn, d) == 1 else
-                             "whole call (%d kernels: %s)" % (launches_per_step(Bn, d),
-                                                             "k_tiles, k_finish" if many_chains(Bn)
-                                                             else "k_verify, k_resid_dot, k_resid_write")),
+                             if launches_per_step(Bn, d, pipelined) == 1 else
+                             "whole call (%d kernels: %s)" % (launches_per_step(Bn, d, pipelined),
+                                                             ", ".join(kernels_of_step(Bn, d, pipelined)))),
                   "duration": "per-call period of 200 back-to-back calls in one CUDA graph "
                               "(events at its two ends only)",
                   "duration_us": 1e3 * ms_call, "algorithmic_bytes": nbytes,
@@ -664,7 +682,7 @@ def main():
                 "hbm_gbs_step": r["roofline"]["algorithmic_bytes"] / (r["ms_step"] * 1e-3) / 1e9,
                 "roofline": r["roofline"], "mean_tau_block": r["taus"]["block"],
                 "mean_tau_sample": r["taus"]["sample"],
-                "gpu_launches": launches_per_step(c["B"], c["d"]) * args.steps}
+                "gpu_launches": launches_per_step(c["B"], c["d"], pipelined) * args.steps}
         subs["sampler"] = sampler_summary(api, dev)
 
     e2e_steps = max(20, min(400, args.steps))
@@ -695,7 +713,7 @@ def main():
                 "d2h_bytes_per_step": d2h,
                 "api": "api.HostStream (pinned [3,B,L,d] window in, accepted_len and y out, "
                        "copy of step i+1 overlapping step i)"},
-        "gpu_launches": launches_per_step(Bn, d) * args.steps,
+        "gpu_launches": launches_per_step(Bn, d, pipelined) * args.steps,
         "clocks": head["clocks"],
         "workloads": subs,
     }

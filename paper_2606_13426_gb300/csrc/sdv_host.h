@@ -21,6 +21,7 @@ constexpr int kK1MinBlocks = 4;
 constexpr int kManyChainMin = 512;
 constexpr int tile_min_blocks(int vpt) { return vpt <= 1 ? 8 : (vpt == 2 ? 6 : 4); }
 constexpr int kFinishThreads = 64;
+constexpr int kFinishWideThreads = 256;
 constexpr int kFinishResidUnroll = 4;
 // Stand-alone acceptance scan: one warp per chain.
 constexpr int kK2Threads = 128;

@@ -828,13 +828,17 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
 // (dynamic, (d + 3)/4 float4), and, with RESID = 1, all kFinishThreads threads write y
 // (launched with 32 threads and leaving the chain state for k_resid_* when RESID = 0).
 // Every output is written after griddep_wait.
-template <typename T, bool VEC4, int RESID>
-__global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
+template <typename T, bool VEC4, int RESID, int NT>
+__global__ void __launch_bounds__(NT) k_finish(VerifyArgs A) {
   __shared__ ChainState cs_s;
-  __shared__ float2 red[kFinishThreads / 32];
+  __shared__ float2 red[NT / 32];
   __shared__ float bcast;
   __shared__ float ell_s[SDV_MAX_L], dn_s[SDV_MAX_L];
+  __shared__ UParams P_s;
+  __shared__ bool haveP_s;
+  __shared__ USampleScratch us;
   extern __shared__ float4 g_s[];  // RESID: the residual's G, drawn once
+  constexpr int RU = NT >= 256 ? kFusedResidUnroll : kFinishResidUnroll;
   const int b = blockIdx.x;
   const int L = A.S.L;
   ScanRegs R;
@@ -861,24 +865,29 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
   if (threadIdx.x < 32) {
     const ScanOut so = scan_decide(A.S, b, R);
     ChainState cs = so.cs;
-    if (cs.kind == kKindResid && A.S.draw_u) {
+    if (NT < 256 && cs.kind == kKindResid && A.S.draw_u) {
+      // a 64-thread CTA: the one-warp U-sampler while warp 1 draws the noise
       const uint32_t wbits = philox_block(seed_of(A.S), (uint32_t)b, 0u, kStreamUSample, 0u).x;
       uint32_t st = cs.status;
       const UParams Q = so.have_P ? so.P : usample_setup(cs.dnorm, fminf(cs.la_res, 0.f));
       cs.U = usample_warp(Q, wbits, &st);
       cs.status = st;
     }
-    if (threadIdx.x == 0) cs_s = cs;
+    if (threadIdx.x == 0) {
+      cs_s = cs;
+      P_s = so.P;
+      haveP_s = so.have_P;
+    }
   } else if (RESID) {
-    prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, kFinishThreads - 32, g_s);
+    prefill_resid_g(seed_of(A.S), b, (A.d + 3) / 4, threadIdx.x - 32, NT - 32, g_s);
   }
   __syncthreads();
-  const ChainState cs = cs_s;
+  ChainState cs = cs_s;
+  if (NT >= 256) draw_u<NT>(A.S, b, cs, haveP_s ? &P_s : nullptr, &us);  // the CTA-wide U-sampler
   const CtaGroup grp{red, &bcast};
   float coef = 0.f;
   if (RESID)
-    coef = residual_coef<T, VEC4, kFinishResidUnroll, 2>((const T*)A.mq, (const T*)A.mp, L, A.d, seed_of(A.S), b,
-                                                         cs, grp, g_s);
+    coef = residual_coef<T, VEC4, RU, 2>((const T*)A.mq, (const T*)A.mp, L, A.d, seed_of(A.S), b, cs, grp, g_s);
   // outputs: after k_tiles has completed, and with it the previous call (see k_tiles)
   griddep_wait();
   for (int i = threadIdx.x; i < L; i += blockDim.x) {
@@ -891,9 +900,8 @@ __global__ void __launch_bounds__(kFinishThreads) k_finish(VerifyArgs A) {
     if (RESID == 0) A.state[b] = cs;
   }
   if (RESID)
-    residual_write<T, VEC4, kFinishResidUnroll, 2>((const T*)A.x, (const T*)A.mq, (const T*)A.mp,
-                                                   (const T*)A.mq_bonus, A.sigma_bonus, L, A.d, seed_of(A.S), b,
-                                                   cs, coef, (T*)A.y, grp, g_s);
+    residual_write<T, VEC4, RU, 2>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, (const T*)A.mq_bonus,
+                                   A.sigma_bonus, L, A.d, seed_of(A.S), b, cs, coef, (T*)A.y, grp, g_s);
 }
 
 // ---------------------------------------------------------------- acceptance scan only
@@ -1200,15 +1208,26 @@ static cudaError_t launch_tiles(const VerifyArgs& A, int B, int L, int vpt, bool
   }
 }
 
+// k_finish: 64 threads per chain, or kFinishWideThreads for rows longer than
+// kFinishMaxGroups groups of four (the pipelined path), whose residual passes and noise
+// a 64-thread CTA would take too long over.
 template <typename T, int RESID>
 static cudaError_t launch_finish(const VerifyArgs& A, int B, bool overlap, cudaStream_t s) {
   const bool vec4 = (A.d % 4 == 0) && aligned(A.x, 4 * sizeof(T)) && aligned(A.mq, 4 * sizeof(T)) &&
                     aligned(A.mp, 4 * sizeof(T)) && (A.y == nullptr || aligned(A.y, 4 * sizeof(T))) &&
                     (A.mq_bonus == nullptr || aligned(A.mq_bonus, 4 * sizeof(T)));
-  const unsigned nt = RESID ? kFinishThreads : 32;
-  const size_t smem = RESID ? sizeof(float4) * (size_t)((A.d + 3) / 4) : 0;
-  if (vec4) return launch_ex(k_finish<T, true, RESID>, (unsigned)B, nt, smem, overlap, A, s);
-  return launch_ex(k_finish<T, false, RESID>, (unsigned)B, nt, smem, overlap, A, s);
+  const int64_t ng = (A.d + 3) / 4;
+  const size_t smem = RESID ? sizeof(float4) * (size_t)ng : 0;
+  if (!RESID) {
+    if (vec4) return launch_ex(k_finish<T, true, 0, 32>, (unsigned)B, 32, 0, overlap, A, s);
+    return launch_ex(k_finish<T, false, 0, 32>, (unsigned)B, 32, 0, overlap, A, s);
+  }
+  if (ng > kFinishMaxGroups) {
+    if (vec4) return launch_ex(k_finish<T, true, 1, kFinishWideThreads>, (unsigned)B, kFinishWideThreads, smem, overlap, A, s);
+    return launch_ex(k_finish<T, false, 1, kFinishWideThreads>, (unsigned)B, kFinishWideThreads, smem, overlap, A, s);
+  }
+  if (vec4) return launch_ex(k_finish<T, true, 1, kFinishThreads>, (unsigned)B, kFinishThreads, smem, overlap, A, s);
+  return launch_ex(k_finish<T, false, 1, kFinishThreads>, (unsigned)B, kFinishThreads, smem, overlap, A, s);
 }
 
 template <typename T>
@@ -1260,16 +1279,14 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
   const int64_t ng = (d + 3) / 4;
-  // Paths.  A pipelined call (overlap) with rows of up to kFinishMaxGroups groups of four
-  // streams with k_tiles and finishes with k_finish, both launched to overlap their
-  // predecessors; with rows of up to kPipeMaxGroups it runs the fused kernel, launched
-  // to overlap its predecessor, with the residual's noise cache in up to 64 KB of
-  // dynamic shared memory (k_finish's 64 threads would write such rows too slowly).
+  // Paths.  A pipelined call (overlap) with rows of up to kPipeMaxGroups groups of four
+  // streams with k_tiles and finishes with k_finish (64 threads per chain; 256 for rows
+  // over kFinishMaxGroups groups), both launched to overlap their predecessors.
   // Otherwise the fused kernel (fewer than kManyChainMin chains) or k_tiles + k_finish
   // (many chains), with the residual of rows longer than the finishing CTA's cache left
   // to k_resid_dot / k_resid_write.
   overlap = overlap && !ratios_only && ng <= kPipeMaxGroups;
-  const bool many = !ratios_only && (overlap ? ng <= kFinishMaxGroups : B >= kManyChainMin);
+  const bool many = !ratios_only && (overlap || B >= kManyChainMin);
   const bool long_rows = !ratios_only && !overlap && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;

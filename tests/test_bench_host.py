@@ -13,9 +13,16 @@ class _Args:
         self.workload, self.mode = workload, mode
 
 
+def test_launches_per_pipelined_call():
+    assert bench.launches_per_step(256, 3072, True) == 2     # k_tiles + k_finish, overlapping
+    assert bench.launches_per_step(64, 16384, True) == 2     # k_finish with 256 threads
+    assert bench.launches_per_step(16, 196608, True) == 3    # too long to overlap: plain path
+    assert bench.kernels_of_step(256, 3072, True) == ["k_tiles", "k_finish"]
+
+
 def test_launches_per_call():
     assert bench.launches_per_step(256, 3072) == 1      # fused kernel
-    assert bench.launches_per_step(64, 16384) == 1      # rows up to 16384 elements stay fused
+    assert bench.launches_per_step(64, 16384) == 3      # plain: fused + long-row dot and write
     assert bench.launches_per_step(16, 196608) == 3     # + long-row dot and write
     assert bench.launches_per_step(1024, 3072) == 2     # k_tiles + k_finish
     assert bench.launches_per_step(1024, 16384) == 4    # k_finish caches up to 4096 elements

@@ -65,6 +65,9 @@ def parse():
                    help="time sdv_verify_ex calls instead of sdv_verify_pipelined")
     p.add_argument("--headline-only", action="store_true",
                    help="skip the latent / high-resolution / sampler sub-results")
+    p.add_argument("--profile", action="store_true",
+                   help="profiler runs: the warm-up and timed steps of the headline workload only "
+                        "(no 200-call pass, steady state, e2e, tau statistics or CPU baseline)")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--skip-cpu", action="store_true")
     return p.parse_args()
@@ -169,25 +172,34 @@ def pipelined_path(d, pipelined):
     return pipelined and (d + 3) // 4 <= PIPE_MAX_GROUPS
 
 
+def wide_finish(B, d, pipelined=False):
+    """Rows of 1025-4096 groups of four finished by a 256-thread k_finish (pipelined
+    calls, or plain calls with fewer than MANY_CHAIN_MIN chains)."""
+    ng = (d + 3) // 4
+    return FINISH_MAX_GROUPS < ng <= PIPE_MAX_GROUPS and (pipelined or not many_chains(B))
+
+
 def long_rows(d, B=0, pipelined=False):
     """Rows whose residual two extra kernels write (longer than the finishing CTA's noise
     cache: the fused kernel's or, on the many-chain path, k_finish's)."""
-    if pipelined_path(d, pipelined):
+    if pipelined_path(d, pipelined) or wide_finish(B, d, pipelined):
         return False
     return (d + 3) // 4 > (FINISH_MAX_GROUPS if many_chains(B) else FUSED_MAX_GROUPS)
 
 
+def _two_kernels(B, d, pipelined):
+    return many_chains(B) or pipelined_path(d, pipelined) or wide_finish(B, d, pipelined)
+
+
 def launches_per_step(B, d, pipelined=False):
     """Kernels one verification call launches: the fused verify kernel, or k_tiles and
-    k_finish (many chains, or a pipelined call), plus the residual dot / write kernels
-    for long rows."""
-    two = many_chains(B) or pipelined_path(d, pipelined)
-    return (2 if two else 1) + (2 if long_rows(d, B, pipelined) else 0)
+    k_finish (many chains, a pipelined call, or rows of 1025-4096 groups), plus the
+    residual dot / write kernels for long rows."""
+    return (2 if _two_kernels(B, d, pipelined) else 1) + (2 if long_rows(d, B, pipelined) else 0)
 
 
 def kernels_of_step(B, d, pipelined=False):
-    two = many_chains(B) or pipelined_path(d, pipelined)
-    names = ["k_tiles", "k_finish"] if two else ["k_verify"]
+    names = ["k_tiles", "k_finish"] if _two_kernels(B, d, pipelined) else ["k_verify"]
     if long_rows(d, B, pipelined):
         names += ["k_resid_dot", "k_resid_write"]
     return names
@@ -466,7 +478,8 @@ def _replay_ms(stream, graphs, reps=1):
     return e0.elapsed_time(e1)
 
 
-def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clocks=None, pipelined=True):
+def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clocks=None, pipelined=True,
+                   profile=False):
     """Timed verification calls on workload `name`: the timed region (steps calls in CUDA
     graph replays, events at its ends), the per-call period of 200 back-to-back calls
     (the roofline's duration), the steady-state period over >= 1 s of replays, and mean
@@ -523,19 +536,22 @@ def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clock
         clocks.start()
         time.sleep(0.3)
     ms_total = _replay_ms(stream, graphs)
-    clk = clocks.stop() if clocks else None
     ms_total = max_over_ranks(ms_total, pg, dev)
     if pg:
         pg.barrier()
     ms_step = ms_total / steps
+    if profile:
+        clk = clocks.stop() if clocks else None
+        return dict(name=name, ms_step=ms_step, clocks=clk)
 
     # the roofline's duration: 200 back-to-back calls in one graph, events at its ends only
     g200 = _graph_of_calls(stream, 200, step)
     _replay_ms(stream, [g200])
     ms_call = min(_replay_ms(stream, [g200]) for _ in range(3)) / 200
-    # steady state: replays of the 200-call graph for >= 1 s
+    # steady state: replays of the 200-call graph for >= 1 s (clocks sampled throughout)
     reps_ss = max(1, int(math.ceil(1000.0 / max(ms_call * 200, 1e-3))))
     ms_ss = _replay_ms(stream, [g200], reps=reps_ss) / (200 * reps_ss)
+    clk = clocks.stop() if clocks else None
 
     taus = {}
     for m in ("block", "sample"):
@@ -663,8 +679,13 @@ def main():
     pipelined = not args.no_pipeline
     clocks = ClockSampler(local)
     head = measure_verify(api, args.workload, Bn, args.mode, args.steps, args.warmup, dev, rank, pg,
-                          clocks, pipelined)
+                          clocks, pipelined, profile=args.profile)
     value = whole_job_rate(world, Bn * L, head["ms_step"] * 1e-3)
+    if args.profile:
+        if rank == 0:
+            print(json.dumps({"metric": "profiler run (not a bench value)", "ms_per_step": head["ms_step"],
+                              "steps": args.steps, "workload": args.workload, "pipelined": pipelined}))
+        return
 
     subs = {}
     if not args.headline_only:

@@ -680,6 +680,12 @@ __device__ __forceinline__ unsigned int ticket_inc(unsigned int* p, unsigned int
   return old;
 }
 
+// The same increment without a result (red): the issuing thread does not wait for it,
+// so a CTA whose last act is counting its tile exits at once.
+__device__ __forceinline__ void ticket_inc_noret(unsigned int* p, unsigned int last) {
+  asm volatile("red.release.gpu.global.inc.u32 [%0], %1;" :: "l"(p), "r"(last) : "memory");
+}
+
 // RESID: 1 = this kernel writes y (the residual's G cached in dynamic shared memory,
 // (d + 3)/4 float4); 0 = it leaves the chain state for k_resid_*.  RU: groups of four
 // elements per thread per residual sweep.
@@ -808,7 +814,7 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
       A.part[tile] = t;
       // release the partial with the chain's count, which wraps to 0 at the chain's
       // last tile; k_finish acquires every partial of the chain by reading that 0
-      ticket_inc(A.ticket + b, (unsigned int)(g * C) - 1u);
+      ticket_inc_noret(A.ticket + b, (unsigned int)(g * C) - 1u);
     }
   }
   if (blockIdx.x == 0) {
@@ -1279,15 +1285,18 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   cudaEvent_t* tev = (ratios_only || !timed) ? nullptr : timing_slot();
   if (tev) timing_record(tev[0], s);
   const int64_t ng = (d + 3) / 4;
-  // Paths.  A pipelined call (overlap) with rows of up to kPipeMaxGroups groups of four
-  // streams with k_tiles and finishes with k_finish (64 threads per chain; 256 for rows
-  // over kFinishMaxGroups groups), both launched to overlap their predecessors.
-  // Otherwise the fused kernel (fewer than kManyChainMin chains) or k_tiles + k_finish
-  // (many chains), with the residual of rows longer than the finishing CTA's cache left
-  // to k_resid_dot / k_resid_write.
+  // Paths (rows in groups of four elements):
+  //  - up to kFusedMaxGroups: the fused kernel for a plain call with fewer than
+  //    kManyChainMin chains; otherwise k_tiles + k_finish (64 threads per chain);
+  //  - up to kPipeMaxGroups: k_tiles + k_finish with 256 threads per chain, except
+  //    for a plain call with many chains (k_tiles + k_finish and the long-row kernels);
+  //  - longer: the fused kernel (or, with many chains, k_tiles + k_finish) without the
+  //    residual, then k_resid_dot / k_resid_write.
+  // A pipelined call launches k_tiles and k_finish to overlap their predecessors.
   overlap = overlap && !ratios_only && ng <= kPipeMaxGroups;
-  const bool many = !ratios_only && (overlap || B >= kManyChainMin);
-  const bool long_rows = !ratios_only && !overlap && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
+  const bool wide = ng > kFinishMaxGroups && ng <= kPipeMaxGroups && (overlap || B < kManyChainMin);
+  const bool many = !ratios_only && (overlap || B >= kManyChainMin || wide);
+  const bool long_rows = !ratios_only && !overlap && !wide && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;
   // the tickets return to zero at the end of every call; a pipelined call relies on

@@ -22,7 +22,7 @@ def test_launches_per_pipelined_call():
 
 def test_launches_per_call():
     assert bench.launches_per_step(256, 3072) == 1      # fused kernel
-    assert bench.launches_per_step(64, 16384) == 3      # plain: fused + long-row dot and write
+    assert bench.launches_per_step(64, 16384) == 2      # plain: k_tiles + 256-thread k_finish
     assert bench.launches_per_step(16, 196608) == 3     # + long-row dot and write
     assert bench.launches_per_step(1024, 3072) == 2     # k_tiles + k_finish
     assert bench.launches_per_step(1024, 16384) == 4    # k_finish caches up to 4096 elements

@@ -91,15 +91,15 @@ def kernel_sources_digest():
     return h.hexdigest()
 
 
-def profile_traffic(workload, full_size):
-    """dram bytes per launch of the fused verify kernel on this workload from its committed
-    ncu summary, if the kernel sources are unchanged since the capture and the batch is
-    the workload's full one (else None)."""
-    path = os.path.join(ROOT, "profiles", "k_verify_%s.md" % workload)
+def profile_traffic(workload, full_size, pipelined=True):
+    """DRAM bytes per call (all of the call's kernels) on this workload from its committed
+    ncu summary (profiles/verify_<workload>_<pipelined|plain>.md), if the kernel sources
+    are unchanged since the capture and the batch is the workload's full one (else None)."""
+    path = os.path.join(ROOT, "profiles", "verify_%s_%s.md" % (workload, "pipelined" if pipelined else "plain"))
     if not full_size or not os.path.exists(path):
         return None
     txt = open(path).read()
-    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    m = re.search(r"traffic_bytes_per_call:\s*([0-9.eE+]+)", txt)
     h = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt)
     if not m or not h:
         return None
@@ -581,7 +581,7 @@ def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clock
                   "duration": "per-call period of 200 back-to-back calls in one CUDA graph "
                               "(events at its two ends only)",
                   "duration_us": 1e3 * ms_call, "algorithmic_bytes": nbytes,
-                  "traffic": profile_traffic(name, Bn == cfg["B"])})
+                  "traffic": profile_traffic(name, Bn == cfg["B"], pipelined)})
 
 
 def measure_e2e(api, host0, Bn, L, d, dt_name, mode, dev, n_steps):

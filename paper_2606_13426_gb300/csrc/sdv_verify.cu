@@ -795,6 +795,68 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
 // (k_tiles: identical partials) at full occupancy, then finishes every chain with
 // a small CTA (k_finish: one warp's scan and U-draw, then the residual row), all
 // chains at once.
+// One tile's 3 VPT 16-byte vectors per thread (a tile is one full sweep: VPT vectors
+// per thread and tensor), issued together with guarded loads, and its (S1, S2)
+// contribution.
+template <int VPT>
+struct TileBuf {
+  uint4 x[VPT], q[VPT], p[VPT];
+};
+
+template <typename T, int VPT>
+__device__ __forceinline__ void tile_issue(const T* __restrict__ x, const T* __restrict__ mq,
+                                           const T* __restrict__ mp, int64_t base, int64_t e0, int64_t e1,
+                                           TileBuf<VPT>& B) {
+  constexpr int V = 16 / (int)sizeof(T);
+  const int64_t v0 = (base + e0) / V;
+  const int nv = (int)((e1 - e0) / V);
+  const uint4* X = reinterpret_cast<const uint4*>(x) + v0;
+  const uint4* Q = reinterpret_cast<const uint4*>(mq) + v0;
+  const uint4* P = reinterpret_cast<const uint4*>(mp) + v0;
+  const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+  for (int u = 0; u < VPT; ++u) {
+    const int vv = threadIdx.x + u * kK1Threads;
+    B.x[u] = vv < nv ? ldg_stream(X + vv) : z;
+  }
+#pragma unroll
+  for (int u = 0; u < VPT; ++u) {
+    const int vv = threadIdx.x + u * kK1Threads;
+    B.q[u] = vv < nv ? ldg_stream(Q + vv) : z;
+  }
+#pragma unroll
+  for (int u = 0; u < VPT; ++u) {
+    const int vv = threadIdx.x + u * kK1Threads;
+    B.p[u] = vv < nv ? ldg_stream(P + vv) : z;
+  }
+}
+
+template <typename T, int VPT>
+__device__ __forceinline__ float2 tile_fma(const TileBuf<VPT>& B) {
+  constexpr int V = 16 / (int)sizeof(T);
+  float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+  for (int u = 0; u < VPT; ++u) {
+    float fx[V], fq[V], fp[V];
+    unpack(B.x[u], fx);
+    unpack(B.q[u], fq);
+    unpack(B.p[u], fp);
+#pragma unroll
+    for (int k = 0; k < V; ++k) {
+      const float dl = fp[k] - fq[k];  // m^p - m^q (zero-filled vectors contribute 0)
+      const float a = fx[k] - fp[k];   // yhat - m^p
+      s1 = fmaf(a, dl, s1);
+      s2 = fmaf(dl, dl, s2);
+    }
+  }
+  return make_float2(s1, s2);
+}
+
+// The stream of the many-chain and pipelined paths: one tile per CTA; its (S1, S2) is
+// stored and counted on its chain (red.release.inc, wrapping to 0 at the chain's last
+// tile).  The FMAs of a tile and their order are those of tile_sums, so the partials
+// equal the fused kernel's.  (Two or four software-pipelined tiles per CTA measured
+// slower: 17.4 / 20.1 us against 16.5 us per pipelined pixel call.)
 template <typename T, bool VEC, int VPT>
 __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(VerifyArgs A) {
   __shared__ float2 red[kK1Threads / 32];
@@ -808,8 +870,15 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   if (j < g) {  // CTA-uniform
     const int64_t e0 = (int64_t)c * A.chunk;
     const int64_t e1 = min(e0 + A.chunk, A.d);
-    const float2 s = tile_sums<T, VEC, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
-    const float2 t = block_sum2<kK1Threads>(s.x, s.y, red);
+    float2 sm;
+    if (VEC) {
+      TileBuf<VPT> B;
+      tile_issue<T, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1, B);
+      sm = tile_fma<T, VPT>(B);
+    } else {
+      sm = tile_sums<T, false, 1>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
+    }
+    const float2 t = block_sum2<kK1Threads>(sm.x, sm.y, red);
     if (threadIdx.x == 0) {
       A.part[tile] = t;
       // release the partial with the chain's count, which wraps to 0 at the chain's
@@ -1148,9 +1217,9 @@ static int validate_window(const void* x, const void* mq, const void* mp, const 
 
 // A launch through cudaLaunchKernelEx: dynamic shared memory (raising the kernel's limit
 // when it passes 48 KB) and, with `overlap`, programmatic stream serialisation.
-template <typename Kern>
+template <typename Kern, typename... Extra>
 static cudaError_t launch_ex(Kern kern, unsigned grid, unsigned threads, size_t smem, bool overlap,
-                             const VerifyArgs& A, cudaStream_t s) {
+                             const VerifyArgs& A, cudaStream_t s, Extra... extra) {
   if (smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -1165,7 +1234,7 @@ static cudaError_t launch_ex(Kern kern, unsigned grid, unsigned threads, size_t 
   at[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = at;
   cfg.numAttrs = overlap ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, A);
+  return cudaLaunchKernelEx(&cfg, kern, A, extra...);
 }
 
 template <typename T, int RESID>

@@ -41,13 +41,14 @@ def test_both_arms_name_the_workload_alike():
 
 
 def test_profile_traffic_lookup():
-    txt = open(os.path.join(bench.ROOT, "profiles", "k_verify_pixel.md")).read()
-    recorded = float(re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt).group(1))
+    path = os.path.join(bench.ROOT, "profiles", "verify_pixel_pipelined.md")
+    txt = open(path).read()
+    recorded = float(re.search(r"traffic_bytes_per_call:\s*([0-9.eE+]+)", txt).group(1))
     digest = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", txt).group(1)
-    got = bench.profile_traffic("pixel", True)
+    got = bench.profile_traffic("pixel", True, True)
     assert got == (recorded if digest == bench.kernel_sources_digest() else None)
-    assert bench.profile_traffic("pixel", False) is None     # not the workload's full batch
-    assert bench.profile_traffic("tiny", True) is None       # no summary for this workload
+    assert bench.profile_traffic("pixel", False, True) is None     # not the workload's full batch
+    assert bench.profile_traffic("tiny", True, True) is None       # no summary for this workload
     # traffic, when reported, is the window plus at most the rejected rows and y
     if got is not None:
         assert 3 * 256 * 8 * 3072 * 4 <= got <= 1.02 * bench.call_bytes(256, 8, 3072, "f32")

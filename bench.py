@@ -581,7 +581,7 @@ def measure_verify(api, name, Bn, mode, steps, warmup, dev, rank, pg=None, clock
                   "duration": "per-call period of 200 back-to-back calls in one CUDA graph "
                               "(events at its two ends only)",
                   "duration_us": 1e3 * ms_call, "algorithmic_bytes": nbytes,
-                  "traffic": profile_traffic(name, Bn == cfg["B"], pipelined)})
+                  "traffic": profile_traffic(name, Bn == cfg["B"], pipelined_path(d, pipelined))})
 
 
 def measure_e2e(api, host0, Bn, L, d, dt_name, mode, dev, n_steps):

@@ -146,3 +146,18 @@ def test_pipelined_calls_in_a_cuda_graph(api):
         torch.cuda.synchronize()
         for i in range(8):
             _same(outs[i], _call(api, sets[i % 4], 300 + i, "block", ws))
+
+
+def test_pipelined_long_rows_run_as_plain_calls(api):
+    """Rows longer than 16384 elements take the plain path even when pipelined (the
+    residual is left to the long-row kernels): identical results to plain calls."""
+    B, L, d = 3, 4, 16388
+    sets = _sets("pixel", 2, B, L, d, False)
+    ws = torch.zeros(api.workspace_bytes(B, L, d, torch.float32), dtype=torch.uint8, device="cuda")
+    piped = [_call(api, sets[i % 2], 500 + i, "block", ws, pipelined=True) for i in range(4)]
+    torch.cuda.synchronize()
+    for i in range(4):
+        ref = _call(api, sets[i % 2], 500 + i, "block", ws)
+        for k in KEYS:
+            a, b = piped[i][k], ref[k]
+            assert torch.equal(torch.nan_to_num(a.float(), nan=7.5), torch.nan_to_num(b.float(), nan=7.5)), k

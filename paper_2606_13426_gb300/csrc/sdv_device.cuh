@@ -51,6 +51,7 @@ constexpr int kGLUnroll = SDV_GL_UNROLL;
 namespace sdv {
 
 // ---------------------------------------------------------------- Philox
+constexpr float kLn2Hi = 0.69314718055994531f;  // log 2 (fp32)
 constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
 constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
 constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
@@ -90,13 +91,21 @@ __device__ __forceinline__ uint4 philox_block(uint64_t seed, uint32_t c0, uint32
   return philox4x32_10(make_uint4(c0, c1, c2, c3), (uint32_t)seed, (uint32_t)(seed >> 32));
 }
 
-// log u for u = (x + 1/2) 2^-32; the upper half goes through 1 - u, which is
-// exact in the integer domain, so log u keeps full relative accuracy near 1.
-// Both forms are evaluated and one selected (no divergence between lanes).
+// log u for u = (x + 1/2) 2^-32 with one logarithm: in the lower half, u = m 2^e with
+// m in [1/2, 1) split off the exponent bits, so log u = (e - 1) log 2 + log1p(2m - 1),
+// 2m - 1 exact; the upper half goes through 1 - u, exact in the integer domain, as
+// log1p(-(1 - u)), so log u keeps full relative accuracy near 1.  The argument and the
+// offset are selected first (no divergence between lanes), then one log1pf.
 __device__ __forceinline__ float log_uniform(uint32_t x) {
-  const float lo = logf(((float)x + 0.5f) * 0x1p-32f);
-  const float hi = log1pf(-(((float)(0xFFFFFFFFu - x) + 0.5f) * 0x1p-32f));
-  return (x < 0x80000000u) ? lo : hi;
+  const float u = ((float)x + 0.5f) * 0x1p-32f;
+  const uint32_t ub = __float_as_uint(u);
+  const float m2 = __uint_as_float((ub & 0x007fffffu) | 0x3f800000u);   // 2m in [1, 2)
+  const float e1 = (float)((int)(ub >> 23) - 127);                      // e - 1
+  const float v = ((float)(0xFFFFFFFFu - x) + 0.5f) * 0x1p-32f;          // 1 - u
+  const bool lower = x < 0x80000000u;
+  const float arg = lower ? m2 - 1.0f : -v;
+  const float base = lower ? e1 * kLn2Hi : 0.0f;
+  return base + log1pf(arg);
 }
 
 // Box-Muller on two words: (r cos 2 pi u1, r sin 2 pi u1), r = sqrt(-2 ln u0).

@@ -168,8 +168,9 @@ def many_chains(B):
 
 
 def pipelined_path(d, pipelined):
-    """Does a pipelined call of row length d take the overlapping k_tiles + k_finish path?"""
-    return pipelined and (d + 3) // 4 <= PIPE_MAX_GROUPS
+    """Does the call take the pipelined path (every kernel launched to overlap its
+    predecessor)?  Every pipelined call does."""
+    return bool(pipelined)
 
 
 def wide_finish(B, d, pipelined=False):
@@ -179,16 +180,16 @@ def wide_finish(B, d, pipelined=False):
     return FINISH_MAX_GROUPS < ng <= PIPE_MAX_GROUPS and (pipelined or not many_chains(B))
 
 
+def _two_kernels(B, d, pipelined):
+    return many_chains(B) or bool(pipelined) or wide_finish(B, d, pipelined)
+
+
 def long_rows(d, B=0, pipelined=False):
     """Rows whose residual two extra kernels write (longer than the finishing CTA's noise
-    cache: the fused kernel's or, on the many-chain path, k_finish's)."""
-    if pipelined_path(d, pipelined) or wide_finish(B, d, pipelined):
+    cache: the fused kernel's, or k_finish's)."""
+    if wide_finish(B, d, pipelined):
         return False
-    return (d + 3) // 4 > (FINISH_MAX_GROUPS if many_chains(B) else FUSED_MAX_GROUPS)
-
-
-def _two_kernels(B, d, pipelined):
-    return many_chains(B) or pipelined_path(d, pipelined) or wide_finish(B, d, pipelined)
+    return (d + 3) // 4 > (FINISH_MAX_GROUPS if _two_kernels(B, d, pipelined) else FUSED_MAX_GROUPS)
 
 
 def launches_per_step(B, d, pipelined=False):

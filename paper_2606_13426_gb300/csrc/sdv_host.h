@@ -33,6 +33,9 @@ constexpr int kK4Threads = 256;
 constexpr int64_t kK4MinChunk = 1024;
 constexpr int64_t kK4MaxChunk = 4096;
 constexpr int64_t kK4TargetCtas = 1024;
+// Pipelined calls: at most this many CTAs per long-row residual kernel (they sit
+// resident, waiting for the chain states, while the next call streams).
+constexpr int64_t kK4PipeCtas = 128;
 // Rows of up to kFusedMaxGroups groups of 4 elements are written by the CTA that
 // finishes the chain inside the fused kernel, kFinishMaxGroups by k_finish on the
 // many-chain path, and kPipeMaxGroups by k_finish on the pipelined path (in each case

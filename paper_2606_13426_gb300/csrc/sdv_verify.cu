@@ -993,6 +993,9 @@ k_resid_dot(const T* __restrict__ mq, const T* __restrict__ mp, int L, int64_t d
             uint64_t seed_v, const uint64_t* __restrict__ seed_dev, const ChainState* __restrict__ state,
             float* __restrict__ part4) {
   __shared__ float2 red[kK4Threads / 32];
+  // pipelined launches: let the next kernel launch now, then wait for the chain states
+  griddep_launch_dependents();
+  griddep_wait();
   const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
   const ChainState cs = state[b];
@@ -1021,6 +1024,9 @@ k_resid_write(const T* __restrict__ x, const T* __restrict__ mq, const T* __rest
               const T* __restrict__ mq_bonus, const float* __restrict__ sigma_bonus, int L,
               int64_t d, int C4, int gpc, uint64_t seed_v, const uint64_t* __restrict__ seed_dev,
               const ChainState* __restrict__ state, const float* __restrict__ part4, T* __restrict__ y) {
+  // pipelined launches: let the next call's stream launch now, then wait for the dots
+  griddep_launch_dependents();
+  griddep_wait();
   const uint64_t seed = seed_dev ? *seed_dev : seed_v;
   const int b = blockIdx.x / C4, c = blockIdx.x - b * C4;
   const ChainState cs = state[b];
@@ -1305,24 +1311,59 @@ static cudaError_t launch_finish(const VerifyArgs& A, int B, bool overlap, cudaS
   return launch_ex(k_finish<T, false, 1, kFinishThreads>, (unsigned)B, kFinishThreads, smem, overlap, A, s);
 }
 
+// A kernel launch through cudaLaunchKernelEx, with programmatic stream serialisation when
+// `overlap`.
+template <typename Kern, typename... Args>
+static cudaError_t launch_pdl(Kern kern, unsigned grid, unsigned threads, bool overlap, cudaStream_t s,
+                              Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads);
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = overlap ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+// The long-row residual kernels: one CTA per chunk of the chain's rejected row.  Plain
+// calls size the chunks for about kK4TargetCtas CTAs (short kernels want many CTAs);
+// pipelined calls for at most kK4PipeCtas, since these kernels wait, resident, for the
+// chain states while the next call streams beside them (few and long CTAs then cost
+// the stream nothing, and their time is hidden).
 template <typename T>
-static void launch_k4(const void* x, const void* mq, const void* mp, const void* mqb,
-                      const float* sb, int B, int L, int64_t d, uint64_t seed, const uint64_t* seed_dev,
-                      const WsLayout& w,
-                      const ChainState* st, float* part4, void* y, cudaStream_t s) {
+static cudaError_t launch_k4(const void* x, const void* mq, const void* mp, const void* mqb,
+                             const float* sb, int B, int L, int64_t d, uint64_t seed, const uint64_t* seed_dev,
+                             const WsLayout& w, const ChainState* st, float* part4, void* y, bool overlap,
+                             cudaStream_t s) {
   const bool vec = (d % 4 == 0) && aligned(x, 4 * sizeof(T)) && aligned(mq, 4 * sizeof(T)) &&
                    aligned(mp, 4 * sizeof(T)) && aligned(y, 4 * sizeof(T)) &&
                    (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
-  const unsigned grid = (unsigned)((int64_t)B * w.C4);
+  int64_t chunk4 = w.chunk4;
+  if (overlap)
+    while ((int64_t)B * ((d + chunk4 - 1) / chunk4) > kK4PipeCtas) chunk4 *= 2;
+  const int C4 = (int)((d + chunk4 - 1) / chunk4);   // <= w.C4: part4 has room
+  const int gpc = (int)(chunk4 / 4);
+  const unsigned grid = (unsigned)((int64_t)B * C4);
+  cudaError_t e;
   if (vec) {
-    k_resid_dot<T, true><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4);
-    k_resid_write<T, true><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                      (const T*)mqb, sb, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4, (T*)y);
+    e = launch_pdl(k_resid_dot<T, true>, grid, kK4Threads, overlap, s, (const T*)mq, (const T*)mp, L, d, C4,
+                   gpc, seed, seed_dev, st, part4);
+    if (e == cudaSuccess)
+      e = launch_pdl(k_resid_write<T, true>, grid, kK4Threads, overlap, s, (const T*)x, (const T*)mq,
+                     (const T*)mp, (const T*)mqb, sb, L, d, C4, gpc, seed, seed_dev, st, (const float*)part4,
+                     (T*)y);
   } else {
-    k_resid_dot<T, false><<<grid, kK4Threads, 0, s>>>((const T*)mq, (const T*)mp, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4);
-    k_resid_write<T, false><<<grid, kK4Threads, 0, s>>>((const T*)x, (const T*)mq, (const T*)mp,
-                                                       (const T*)mqb, sb, L, d, w.C4, w.chunk4 / 4, seed, seed_dev, st, part4, (T*)y);
+    e = launch_pdl(k_resid_dot<T, false>, grid, kK4Threads, overlap, s, (const T*)mq, (const T*)mp, L, d, C4,
+                   gpc, seed, seed_dev, st, part4);
+    if (e == cudaSuccess)
+      e = launch_pdl(k_resid_write<T, false>, grid, kK4Threads, overlap, s, (const T*)x, (const T*)mq,
+                     (const T*)mp, (const T*)mqb, sb, L, d, C4, gpc, seed, seed_dev, st, (const float*)part4,
+                     (T*)y);
   }
+  return e;
 }
 
 // Enqueue the whole step (or, with ratios_only, the log-ratio pass) for validated args.
@@ -1359,13 +1400,13 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   //    kManyChainMin chains; otherwise k_tiles + k_finish (64 threads per chain);
   //  - up to kPipeMaxGroups: k_tiles + k_finish with 256 threads per chain, except
   //    for a plain call with many chains (k_tiles + k_finish and the long-row kernels);
-  //  - longer: the fused kernel (or, with many chains, k_tiles + k_finish) without the
-  //    residual, then k_resid_dot / k_resid_write.
-  // A pipelined call launches k_tiles and k_finish to overlap their predecessors.
-  overlap = overlap && !ratios_only && ng <= kPipeMaxGroups;
+  //  - longer: the fused kernel (or, with many chains or pipelined, k_tiles +
+  //    k_finish) without the residual, then k_resid_dot / k_resid_write.
+  // A pipelined call launches every one of its kernels to overlap its predecessor.
+  overlap = overlap && !ratios_only;
   const bool wide = ng > kFinishMaxGroups && ng <= kPipeMaxGroups && (overlap || B < kManyChainMin);
   const bool many = !ratios_only && (overlap || B >= kManyChainMin || wide);
-  const bool long_rows = !ratios_only && !overlap && !wide && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
+  const bool long_rows = !ratios_only && !wide && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;
   // the tickets return to zero at the end of every call; a pipelined call relies on
@@ -1406,10 +1447,15 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   }
   if (long_rows) {
     float* part4 = (float*)(ws + w.part4_off);
-    if (f32)
-      launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev, w, A.state, part4, y_out, s);
-    else
-      launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev, w, A.state, part4, y_out, s);
+    e = f32 ? launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev,
+                               w, A.state, part4, y_out, overlap, s)
+            : launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed,
+                                       seed_dev, w, A.state, part4, y_out, overlap, s);
+    if (e != cudaSuccess) {
+      g_last_cuda_error = (int)e;
+      cudaGetLastError();
+      return SDV_ECUDA;
+    }
     rc = check_launch();
   }
   if (tev) timing_record(tev[2], s);

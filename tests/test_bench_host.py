@@ -16,7 +16,7 @@ class _Args:
 def test_launches_per_pipelined_call():
     assert bench.launches_per_step(256, 3072, True) == 2     # k_tiles + k_finish, overlapping
     assert bench.launches_per_step(64, 16384, True) == 2     # k_finish with 256 threads
-    assert bench.launches_per_step(16, 196608, True) == 3    # too long to overlap: plain path
+    assert bench.launches_per_step(16, 196608, True) == 4    # + the long-row kernels, all overlapping
     assert bench.kernels_of_step(256, 3072, True) == ["k_tiles", "k_finish"]
 
 

@@ -1342,8 +1342,8 @@ static cudaError_t launch_k4(const void* x, const void* mq, const void* mp, cons
                    aligned(mp, 4 * sizeof(T)) && aligned(y, 4 * sizeof(T)) &&
                    (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
   int64_t chunk4 = w.chunk4;
-  if (overlap)
-    while ((int64_t)B * ((d + chunk4 - 1) / chunk4) > kK4PipeCtas) chunk4 *= 2;
+  if (overlap)  // at least one chunk per chain
+    while (chunk4 < d && (int64_t)B * ((d + chunk4 - 1) / chunk4) > kK4PipeCtas) chunk4 *= 2;
   const int C4 = (int)((d + chunk4 - 1) / chunk4);   // <= w.C4: part4 has room
   const int gpc = (int)(chunk4 / 4);
   const unsigned grid = (unsigned)((int64_t)B * C4);

@@ -165,3 +165,15 @@ def test_pipelined_long_rows(api):
     o = oracle_for(inp, 505, OV.MODE_BLOCK)
     g = {k: v.cpu().numpy() for k, v in piped[5].items()}
     compare(g, o, OV.MODE_BLOCK, "f32")
+
+
+def test_pipelined_long_rows_many_chains(api):
+    """Many chains with long rows: the residual kernels keep one chunk per chain at least
+    (more chains than their CTA budget)."""
+    B, L, d = 520, 2, 16388
+    sets = _sets("pixel", 1, B, L, d, False)
+    ws = torch.zeros(api.workspace_bytes(B, L, d, torch.float32), dtype=torch.uint8, device="cuda")
+    piped = [_call(api, sets[0], 700 + i, "sample", ws, pipelined=True) for i in range(2)]
+    torch.cuda.synchronize()
+    for i in range(2):
+        _same(piped[i], _call(api, sets[0], 700 + i, "sample", ws))

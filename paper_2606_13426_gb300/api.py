@@ -34,7 +34,9 @@ def workspace_bytes(B_, L, d, dtype=torch.float32):
 
 
 def make_workspace(B_, L, d, dtype=torch.float32, device="cuda"):
-    return torch.empty(max(workspace_bytes(B_, L, d, dtype), 256), dtype=torch.uint8, device=device)
+    """A zeroed workspace (its counters must start at zero for pipelined calls; every call
+    leaves them at zero)."""
+    return torch.zeros(max(workspace_bytes(B_, L, d, dtype), 256), dtype=torch.uint8, device=device)
 
 
 def _sigma_args(sigma, Bn, L):

@@ -180,8 +180,12 @@ def wide_finish(B, d, pipelined=False):
     return FINISH_MAX_GROUPS < ng <= PIPE_MAX_GROUPS and (pipelined or not many_chains(B))
 
 
+# Plain calls with fewer chains run the fused kernel (the library's kFusedMaxChains).
+FUSED_MAX_CHAINS = 64
+
+
 def _two_kernels(B, d, pipelined):
-    return many_chains(B) or bool(pipelined) or wide_finish(B, d, pipelined)
+    return B >= FUSED_MAX_CHAINS or bool(pipelined) or wide_finish(B, d, pipelined)
 
 
 def long_rows(d, B=0, pipelined=False):

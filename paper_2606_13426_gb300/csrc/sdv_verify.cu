@@ -1397,7 +1397,7 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   const int64_t ng = (d + 3) / 4;
   // Paths (rows in groups of four elements):
   //  - up to kFusedMaxGroups: the fused kernel for a plain call with fewer than
-  //    kManyChainMin chains; otherwise k_tiles + k_finish (64 threads per chain);
+  //    kFusedMaxChains chains; otherwise k_tiles + k_finish (64 threads per chain);
   //  - up to kPipeMaxGroups: k_tiles + k_finish with 256 threads per chain, except
   //    for a plain call with many chains (k_tiles + k_finish and the long-row kernels);
   //  - longer: the fused kernel (or, with many chains or pipelined, k_tiles +
@@ -1405,7 +1405,7 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   // A pipelined call launches every one of its kernels to overlap its predecessor.
   overlap = overlap && !ratios_only;
   const bool wide = ng > kFinishMaxGroups && ng <= kPipeMaxGroups && (overlap || B < kManyChainMin);
-  const bool many = !ratios_only && (overlap || B >= kManyChainMin || wide);
+  const bool many = !ratios_only && (overlap || B >= kFusedMaxChains || wide);
   const bool long_rows = !ratios_only && !wide && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;

@@ -21,7 +21,8 @@ def test_launches_per_pipelined_call():
 
 
 def test_launches_per_call():
-    assert bench.launches_per_step(256, 3072) == 1      # fused kernel
+    assert bench.launches_per_step(32, 3072) == 1       # fused kernel (fewer than 64 chains)
+    assert bench.launches_per_step(256, 3072) == 2      # k_tiles + k_finish
     assert bench.launches_per_step(64, 16384) == 2      # plain: k_tiles + 256-thread k_finish
     assert bench.launches_per_step(16, 196608) == 3     # + long-row dot and write
     assert bench.launches_per_step(1024, 3072) == 2     # k_tiles + k_finish

@@ -1337,7 +1337,7 @@ template <typename T>
 static cudaError_t launch_k4(const void* x, const void* mq, const void* mp, const void* mqb,
                              const float* sb, int B, int L, int64_t d, uint64_t seed, const uint64_t* seed_dev,
                              const WsLayout& w, const ChainState* st, float* part4, void* y, bool overlap,
-                             cudaStream_t s) {
+                             bool pdl, cudaStream_t s) {
   const bool vec = (d % 4 == 0) && aligned(x, 4 * sizeof(T)) && aligned(mq, 4 * sizeof(T)) &&
                    aligned(mp, 4 * sizeof(T)) && aligned(y, 4 * sizeof(T)) &&
                    (mqb == nullptr || aligned(mqb, 4 * sizeof(T)));
@@ -1349,17 +1349,17 @@ static cudaError_t launch_k4(const void* x, const void* mq, const void* mp, cons
   const unsigned grid = (unsigned)((int64_t)B * C4);
   cudaError_t e;
   if (vec) {
-    e = launch_pdl(k_resid_dot<T, true>, grid, kK4Threads, overlap, s, (const T*)mq, (const T*)mp, L, d, C4,
+    e = launch_pdl(k_resid_dot<T, true>, grid, kK4Threads, pdl, s, (const T*)mq, (const T*)mp, L, d, C4,
                    gpc, seed, seed_dev, st, part4);
     if (e == cudaSuccess)
-      e = launch_pdl(k_resid_write<T, true>, grid, kK4Threads, overlap, s, (const T*)x, (const T*)mq,
+      e = launch_pdl(k_resid_write<T, true>, grid, kK4Threads, pdl, s, (const T*)x, (const T*)mq,
                      (const T*)mp, (const T*)mqb, sb, L, d, C4, gpc, seed, seed_dev, st, (const float*)part4,
                      (T*)y);
   } else {
-    e = launch_pdl(k_resid_dot<T, false>, grid, kK4Threads, overlap, s, (const T*)mq, (const T*)mp, L, d, C4,
+    e = launch_pdl(k_resid_dot<T, false>, grid, kK4Threads, pdl, s, (const T*)mq, (const T*)mp, L, d, C4,
                    gpc, seed, seed_dev, st, part4);
     if (e == cudaSuccess)
-      e = launch_pdl(k_resid_write<T, false>, grid, kK4Threads, overlap, s, (const T*)x, (const T*)mq,
+      e = launch_pdl(k_resid_write<T, false>, grid, kK4Threads, pdl, s, (const T*)x, (const T*)mq,
                      (const T*)mp, (const T*)mqb, sb, L, d, C4, gpc, seed, seed_dev, st, (const float*)part4,
                      (T*)y);
   }
@@ -1433,11 +1433,15 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   int rc = check_launch();
   if (rc != SDV_OK) return rc;
   if (tev) timing_record(tev[1], s);
+  // The kernels after the first of a call are always launched to overlap their
+  // predecessor within the call: k_finish reads nothing before every k_tiles CTA has
+  // counted its tile, and the residual kernels wait for their inputs at their start;
+  // only the first kernel's overlap with the previous call needs the pipelined contract.
   if (many) {
     if (long_rows)
-      e = f32 ? launch_finish<float, 0>(A, B, overlap, s) : launch_finish<__nv_bfloat16, 0>(A, B, overlap, s);
+      e = f32 ? launch_finish<float, 0>(A, B, true, s) : launch_finish<__nv_bfloat16, 0>(A, B, true, s);
     else
-      e = f32 ? launch_finish<float, 1>(A, B, overlap, s) : launch_finish<__nv_bfloat16, 1>(A, B, overlap, s);
+      e = f32 ? launch_finish<float, 1>(A, B, true, s) : launch_finish<__nv_bfloat16, 1>(A, B, true, s);
     if (e != cudaSuccess) {
       g_last_cuda_error = (int)e;
       cudaGetLastError();
@@ -1448,9 +1452,9 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   if (long_rows) {
     float* part4 = (float*)(ws + w.part4_off);
     e = f32 ? launch_k4<float>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed, seed_dev,
-                               w, A.state, part4, y_out, overlap, s)
+                               w, A.state, part4, y_out, overlap, true, s)
             : launch_k4<__nv_bfloat16>(x_draft, mu_target, mu_draft, mu_target_bonus, sigma_bonus, B, L, d, seed,
-                                       seed_dev, w, A.state, part4, y_out, overlap, s);
+                                       seed_dev, w, A.state, part4, y_out, overlap, true, s);
     if (e != cudaSuccess) {
       g_last_cuda_error = (int)e;
       cudaGetLastError();

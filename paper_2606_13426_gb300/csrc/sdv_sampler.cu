@@ -557,10 +557,10 @@ struct SamplerCtl {
   uint64_t seed_r;
   int32_t r;
   uint32_t active;
-  uint32_t done;  // chains whose update finished this round
+  uint32_t done;  // k_round_update CTAs that finished this round
 };
 
-// End of a round (the last chain's CTA, after every chain's ticket): advance the
+// End of a round (the k_round_update CTA holding the round's last ticket): advance the
 // round counter and seed, reset the round's counters, and (inside the round graph)
 // keep the loop going while a chain is active and fewer than max_rounds rounds ran.
 __device__ __forceinline__ void close_round(SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
@@ -574,52 +574,67 @@ __device__ __forceinline__ void close_round(SamplerCtl* ctl, uint64_t seed, int 
   if (in_loop) cudaGraphSetConditional(h, more ? 1u : 0u);
 }
 
-// Round bookkeeping, one CTA per chain: the emitted state, the score cache, k, the next
-// window length and the statistics; counts the chains that remain active, and the
-// CTA holding the round's last ticket closes the round (close_round).
+// Round bookkeeping, one warp per chain and kUpdateChains chains per CTA: the emitted
+// state, the score cache, k, the next window length and the statistics; each CTA adds
+// its chains that remain active with one atomic, and the CTA holding the round's last
+// ticket closes the round (close_round).  (One CTA per chain made 1024 same-address
+// atomics per round, and that serialisation cost most of the kernel's time.)
 // VEC: d % 4 == 0 (workspace rows are then 16-byte aligned).
+constexpr int kUpdateChains = 8;
+
 template <bool VEC>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(32 * kUpdateChains)
 k_round_update(const int32_t* __restrict__ acc, const float* __restrict__ y_out,
-               const float* __restrict__ x_draft, const float* __restrict__ sc_all, int L, int64_t d,
+               const float* __restrict__ x_draft, const float* __restrict__ sc_all, int B, int L, int64_t d,
                int K, float* y, float* s_cache, int32_t* kk, int32_t* gam, int32_t* rounds,
                int32_t* tau_sum, SamplerCtl* ctl, uint64_t seed, int max_rounds, int in_loop,
                cudaGraphConditionalHandle h) {
-  const int b = blockIdx.x;
-  const int g = gam[b];
-  const int k = kk[b];
-  __syncthreads();  // every thread has read k and gamma before thread 0 updates them
-  const int tau = acc[b] + 1;
-  if (g > 0) {
-    const bool end = (tau == g + 1) && (k + g >= K);  // no bonus step past the end of sampling
-    const float* ysrc = end ? x_draft + ((int64_t)b * L + g - 1) * d : y_out + (int64_t)b * d;
-    const float* ssrc = sc_all + ((int64_t)b * (L + 1) + min(tau, g)) * d;
-    if (VEC) {
-      const float4* ys4 = reinterpret_cast<const float4*>(ysrc);
-      const float4* ss4 = reinterpret_cast<const float4*>(ssrc);
-      float4* yd4 = reinterpret_cast<float4*>(y + (int64_t)b * d);
-      float4* sd4 = reinterpret_cast<float4*>(s_cache + (int64_t)b * d);
-      for (int64_t i = threadIdx.x; i < d / 4; i += blockDim.x) {
-        yd4[i] = ys4[i];
-        sd4[i] = ss4[i];
+  __shared__ unsigned int act_s[kUpdateChains];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * kUpdateChains + w;
+  unsigned int act = 0u;
+  if (b < B) {
+    const int g = gam[b];
+    const int k = kk[b];
+    __syncwarp();  // every lane has read k and gamma before lane 0 updates them
+    const int tau = acc[b] + 1;
+    if (g > 0) {
+      const bool end = (tau == g + 1) && (k + g >= K);  // no bonus step past the end of sampling
+      const float* ysrc = end ? x_draft + ((int64_t)b * L + g - 1) * d : y_out + (int64_t)b * d;
+      const float* ssrc = sc_all + ((int64_t)b * (L + 1) + min(tau, g)) * d;
+      if (VEC) {
+        const float4* ys4 = reinterpret_cast<const float4*>(ysrc);
+        const float4* ss4 = reinterpret_cast<const float4*>(ssrc);
+        float4* yd4 = reinterpret_cast<float4*>(y + (int64_t)b * d);
+        float4* sd4 = reinterpret_cast<float4*>(s_cache + (int64_t)b * d);
+        for (int64_t i = lane; i < d / 4; i += 32) {
+          yd4[i] = ys4[i];
+          sd4[i] = ss4[i];
+        }
+      } else {
+        for (int64_t i = lane; i < d; i += 32) {
+          y[(int64_t)b * d + i] = ysrc[i];
+          s_cache[(int64_t)b * d + i] = ssrc[i];
+        }
       }
-    } else {
-      for (int64_t i = threadIdx.x; i < d; i += blockDim.x) {
-        y[(int64_t)b * d + i] = ysrc[i];
-        s_cache[(int64_t)b * d + i] = ssrc[i];
+      if (lane == 0) {
+        const int kn = min(k + tau, K);
+        kk[b] = kn;
+        const int gn = kn < K ? min(L, K - kn) : 0;
+        gam[b] = gn;
+        rounds[b] += 1;
+        tau_sum[b] += tau;
+        act = gn > 0 ? 1u : 0u;
       }
     }
   }
+  if (lane == 0) act_s[w] = act;
+  __syncthreads();
   if (threadIdx.x == 0) {
-    if (g > 0) {
-      const int kn = min(k + tau, K);
-      kk[b] = kn;
-      const int gn = kn < K ? min(L, K - kn) : 0;
-      gam[b] = gn;
-      rounds[b] += 1;
-      tau_sum[b] += tau;
-      if (gn > 0) atomicAdd(&ctl->active, 1u);
-    }
+    unsigned int n = 0u;
+#pragma unroll
+    for (int i = 0; i < kUpdateChains; ++i) n += act_s[i];
+    if (n) atomicAdd(&ctl->active, n);
     if (ticket_acq_rel(&ctl->done) == gridDim.x - 1) close_round(ctl, seed, max_rounds, in_loop, h);
   }
 }
@@ -898,11 +913,13 @@ static int enqueue_round(const SamplerRun& R, cudaStream_t cs, int max_rounds, b
                       R.vws, R.vws_bytes, false, cs);
   if (rc != SDV_OK) return rc;
   if (d % 4 == 0)
-    k_round_update<true><<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam,
-                                            R.rounds, R.tsum, R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
+    k_round_update<true><<<(B + kUpdateChains - 1) / kUpdateChains, 32 * kUpdateChains, 0, cs>>>(
+        R.acc, R.yo, R.xd, R.scall, B, L, d, R.K, R.y, R.sc, R.kk, R.gam, R.rounds, R.tsum, R.ctl, R.seed,
+        max_rounds, loop ? 1 : 0, handle);
   else
-    k_round_update<false><<<B, 256, 0, cs>>>(R.acc, R.yo, R.xd, R.scall, L, d, R.K, R.y, R.sc, R.kk, R.gam,
-                                             R.rounds, R.tsum, R.ctl, R.seed, max_rounds, loop ? 1 : 0, handle);
+    k_round_update<false><<<(B + kUpdateChains - 1) / kUpdateChains, 32 * kUpdateChains, 0, cs>>>(
+        R.acc, R.yo, R.xd, R.scall, B, L, d, R.K, R.y, R.sc, R.kk, R.gam, R.rounds, R.tsum, R.ctl, R.seed,
+        max_rounds, loop ? 1 : 0, handle);
   return launch_check();
 }
 

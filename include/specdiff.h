@@ -78,9 +78,10 @@ const char *sdv_strerror(int code);
 int sdv_last_cuda_error(void);
 
 /*
- * Bytes of device workspace sdv_verify / sdv_verify_ex / sdv_log_ratios need
- * for (B, L, d, dtype); 0 for invalid sizes.  The caller allocates it (any
- * 256-byte aligned device buffer) and may reuse it across calls on one stream.
+ * Bytes of device workspace sdv_verify / sdv_verify_ex / sdv_log_ratios /
+ * sdv_verify_pipelined need for (B, L, d, dtype); 0 for invalid sizes.  The caller
+ * allocates it (any 256-byte aligned device buffer, its contents arbitrary) and may
+ * reuse it across calls of any sizes on one stream.
  */
 size_t sdv_workspace_bytes(int B, int L, int64_t d, int dtype);
 
@@ -160,19 +161,18 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  * decomposition-res, u-sample): log ratios, accepted lengths and status equal
  * sdv_verify_ex's bit for bit; U and y agree within the library's accuracy (rows of
  * up to 4096 elements finish in a 64-thread CTA with the one-warp U-sampler).
- * Preconditions (the caller's promise; nothing checks them):
- *   - the window (x_draft, mu_target, mu_draft, sigma, L_eff, mu_target_bonus,
- *     sigma_bonus) is not written by earlier work on `stream` that may still be
- *     running: the previous kernel, and the earlier calls of a run of pipelined
- *     calls (the window is read while they finish);
- *   - the workspace's counters are zero: the workspace is fresh from a
- *     cudaMemset to 0, or was last used by a completed call of this library
- *     (every call leaves them at zero).
+ * Precondition (the caller's promise; nothing checks it): the window (x_draft,
+ * mu_target, mu_draft, sigma, L_eff, mu_target_bonus, sigma_bonus) is not written by
+ * earlier work on `stream` that may still be running: the previous kernel, and the
+ * earlier calls of a run of pipelined calls (the window is read while they finish).
+ * The workspace needs no preparation: each tile partial is stored with a tag of its
+ * call, and the finishing kernel waits for the whole stream of its call when it reads
+ * a partial without that tag.
  * Outputs are written only after the previous call on `stream` has written its own,
- * so consecutive calls may share output buffers.  The overlap applies to rows of up
- * to 16384 elements; longer rows run exactly as sdv_verify_ex.  Same arguments,
- * return codes and ownership as sdv_verify_ex; the workspace must not be shared with
- * calls on other streams.
+ * so consecutive calls may share output buffers.  Rows longer than 16384 elements
+ * add two residual kernels, which overlap the next call's stream too.  Same
+ * arguments, return codes and ownership as sdv_verify_ex; the workspace must not be
+ * shared with calls on other streams.
  */
 int sdv_verify_pipelined(const void *x_draft, const void *mu_target, const void *mu_draft,
                          const float *sigma, int64_t sigma_stride_b,

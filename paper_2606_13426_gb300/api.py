@@ -34,8 +34,7 @@ def workspace_bytes(B_, L, d, dtype=torch.float32):
 
 
 def make_workspace(B_, L, d, dtype=torch.float32, device="cuda"):
-    """A zeroed workspace (its counters must start at zero for pipelined calls; every call
-    leaves them at zero)."""
+    """A workspace for calls of up to (B_, L, d) (zeroed, though no call needs that)."""
     return torch.zeros(max(workspace_bytes(B_, L, d, dtype), 256), dtype=torch.uint8, device=device)
 
 

@@ -24,7 +24,10 @@ constexpr int kManyChainMin = 512;
 // k_finish (measured per call, pixel rows: B = 16 18.5 against 22.5 us, B = 64 24.9
 // against 24.3, B = 256 38.2 against 34.8 in block mode).
 constexpr int kFusedMaxChains = 64;
-constexpr int tile_min_blocks(int vpt) { return vpt <= 1 ? 8 : (vpt == 2 ? 6 : 4); }
+// Three vectors per thread fit 48 registers, so that four k_tiles CTAs still leave
+// room for two 64-thread k_finish CTAs of the previous pipelined call on the same SM
+// (pipelined pixel rows 16.4 -> 16.3 us per call in block mode, 16.2 -> 15.7 in sample).
+constexpr int tile_min_blocks(int vpt) { return vpt <= 1 ? 8 : (vpt == 2 ? 6 : (vpt == 3 ? 5 : 4)); }
 constexpr int kFinishThreads = 64;
 constexpr int kFinishWideThreads = 256;
 constexpr int kFinishResidUnroll = 4;
@@ -77,7 +80,9 @@ struct ChainState {
 };
 
 struct ScanArgs {
-  const float2* part;
+  const float2* part;     // fused kernel: [B, L, C] (S1, S2) per tile
+  const uint64_t* tpart;  // k_tiles: [B, L, C] pairs of words (S1 | tag << 32, S2 | tag << 32)
+  uint32_t tag;           // this call's tag of its k_tiles partials (never 0)
   int C;
   const float* sigma;
   int64_t sstride;
@@ -108,6 +113,8 @@ struct WsLayout {
   int C1;          // K1 tiles per row
   int64_t chunk4;  // K4 elements per tile
   int C4;          // K4 tiles per chain
+  // tickets [B] u32 (fused kernel), tile partials [B, L, C1] 16 bytes each (the fused
+  // kernel's float2 or k_tiles' tagged pair of words), chain states, long-row partials
   size_t ticket_off, part_off, state_off, part4_off, total;
 };
 

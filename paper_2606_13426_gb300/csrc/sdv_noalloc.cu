@@ -51,8 +51,9 @@ extern "C" int sdv_verify_noalloc(const void* x_draft, const void* mu_target, co
     sdv::set_last_cuda_error((int)cudaGetLastError());
     return SDV_ECUDA;
   }
-  // The tickets that must start at zero are cleared by the call itself (a memset on
-  // `stream`); everything else in the workspace is written before it is read.
+  // The tickets of the fused kernel, which must start at zero, are cleared by the call
+  // itself (a memset on `stream`); k_tiles' partials carry the call's tag; everything
+  // else in the workspace is written before it is read.
   return sdv_verify(x_draft, mu_target, mu_draft, sigma, sigma_stride_b, B, L, d, dtype, seed, mode,
                     accepted_len, y_out, log_ratio_out, delta_norm_out, status_out, scratch,
                     (size_t)SDV_NOALLOC_SCRATCH_BYTES, stream);

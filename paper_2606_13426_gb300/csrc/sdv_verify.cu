@@ -1,7 +1,7 @@
 // sdv_verify.cu - verification step of speculative diffusion sampling on sm_103a.
 //
-// One sdv_verify call launches (on the caller's stream) a counter reset and ONE
-// fused kernel, k_verify:
+// One sdv_verify call with few chains launches (on the caller's stream) a counter
+// reset and ONE fused kernel, k_verify:
 //   * every CTA streams one tile (chain b, step j, chunk c) of x, m^q and m^p once
 //     with 16-byte loads and reduces S1 = sum (x - m^p)(m^p - m^q) and
 //     S2 = sum (m^p - m^q)^2 (App. "Density ratio calculations": Z^T Delta =
@@ -15,12 +15,14 @@
 // Chains finish at staggered times, so the latency-bound per-chain work overlaps
 // the streaming of other chains.  Rows longer than kFusedMaxGroups groups of four
 // elements are written by two extra kernels (k_resid_dot, k_resid_write) spread
-// over many CTAs.  With many chains (B >= kManyChainMin) the same tiles are
-// streamed by k_tiles and every chain is finished by a small CTA of k_finish.
+// over many CTAs.  With many chains (B >= kFusedMaxChains), and in pipelined calls,
+// the same tiles are streamed by k_tiles (each partial stored with the call's tag)
+// and every chain is finished by a small CTA of k_finish.
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -218,12 +220,14 @@ struct ScanRegs {
   float ell[2], dn[2], S1[2], S2[2], sg[2];
   int g;         // window length gamma_k, clamped to [0, L]
   bool any_bad;  // a non-finite ratio, norm or sigma
+  bool stale;    // a k_tiles partial without this call's tag (not yet visible)
 };
 
 // Loads chain b's ell_j and |Delta_j|: from the tile partials (S1, S2 of every tile of
-// the row, read through L2) and sigma, or from given arrays.  Called by a full warp;
-// reads only.
-__device__ ScanRegs scan_load(const ScanArgs& A, int b) {
+// the row, read through L2) and sigma, or from given arrays.  k_tiles partials carry the
+// call's tag in each 8-byte word (written whole); with check_tags, R.stale reports a
+// word whose tag is not this call's.  Called by a full warp; reads only.
+__device__ ScanRegs scan_load(const ScanArgs& A, int b, bool check_tags = true) {
   const unsigned FULL = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   const int L = A.L;
@@ -231,21 +235,33 @@ __device__ ScanRegs scan_load(const ScanArgs& A, int b) {
   // window length gamma_k, clamped to [0, L] (device data the host cannot check)
   R.g = A.L_eff ? max(0, min(A.L_eff[b], L)) : L;
   const int nseg = (L + 31) >> 5;
-  bool bad = false;
+  bool bad = false, stale = false;
 #pragma unroll
   for (int q = 0; q < 2; ++q) {
     const int j = lane + 32 * q;
     R.ell[q] = 0.f; R.dn[q] = 0.f; R.S1[q] = 0.f; R.S2[q] = 0.f; R.sg[q] = 1.f;
     if (q < nseg && j < R.g) {
-      if (A.part) {
-        // partials written by other CTAs of this grid: read through L2
-        const float2* p = A.part + ((int64_t)b * L + j) * A.C;
+      if (A.part || A.tpart) {
+        // partials written by other CTAs: read through L2, summed over the row's tiles
+        // in tile order
         float a1 = 0.f, a2 = 0.f;
+        if (A.tpart) {
+          const ulonglong2* p = reinterpret_cast<const ulonglong2*>(A.tpart) + ((int64_t)b * L + j) * A.C;
 #pragma unroll 4
-        for (int c = 0; c < A.C; ++c) {
-          const float2 t = __ldcg(p + c);
-          a1 += t.x;
-          a2 += t.y;
+          for (int c = 0; c < A.C; ++c) {
+            const ulonglong2 t = __ldcg(p + c);
+            if (check_tags && ((uint32_t)(t.x >> 32) != A.tag || (uint32_t)(t.y >> 32) != A.tag)) stale = true;
+            a1 += __uint_as_float((uint32_t)t.x);
+            a2 += __uint_as_float((uint32_t)t.y);
+          }
+        } else {
+          const float2* p = A.part + ((int64_t)b * L + j) * A.C;
+#pragma unroll 4
+          for (int c = 0; c < A.C; ++c) {
+            const float2 t = __ldcg(p + c);
+            a1 += t.x;
+            a2 += t.y;
+          }
         }
         const float s = A.sigma[(int64_t)b * A.sstride + j];
         R.S1[q] = a1; R.S2[q] = a2; R.sg[q] = s;
@@ -261,6 +277,7 @@ __device__ ScanRegs scan_load(const ScanArgs& A, int b) {
     }
   }
   R.any_bad = __any_sync(FULL, bad);
+  R.stale = __any_sync(FULL, stale);
   return R;
 }
 
@@ -663,8 +680,9 @@ struct VerifyArgs {
   int64_t d;
   int64_t chunk;
   void* y;
-  float2* part;          // [B, L, C] tile partials (also read through S.part)
-  unsigned int* ticket;  // [B], zero at launch
+  float2* part;          // [B, L, C] fused kernel's tile partials (also read through S.part)
+  uint64_t* tpart;       // the same slots as k_tiles' tagged partials (read through S.tpart)
+  unsigned int* ticket;  // [B], zero at launch of the fused kernel
   ChainState* state;     // [B]; written when the residual row is left to k_resid_*
   ScanArgs S;
 };
@@ -680,12 +698,6 @@ __device__ __forceinline__ unsigned int ticket_inc(unsigned int* p, unsigned int
   return old;
 }
 
-// The same increment without a result (red): the issuing thread does not wait for it,
-// so a CTA whose last act is counting its tile exits at once.
-__device__ __forceinline__ void ticket_inc_noret(unsigned int* p, unsigned int last) {
-  asm volatile("red.release.gpu.global.inc.u32 [%0], %1;" :: "l"(p), "r"(last) : "memory");
-}
-
 // RESID: 1 = this kernel writes y (the residual's G cached in dynamic shared memory,
 // (d + 3)/4 float4); 0 = it leaves the chain state for k_resid_*.  RU: groups of four
 // elements per thread per residual sweep.
@@ -693,8 +705,8 @@ __device__ __forceinline__ void ticket_inc_noret(unsigned int* p, unsigned int l
 // Ordering against the previous kernel on the stream (see griddep_wait): this kernel
 // writes nothing the previous one may read except its own outputs, and those only after
 // griddep_wait; a finishing CTA triggers its dependents once it has read the chain's
-// partials, the only workspace data that the next call overwrites; the tickets return
-// to zero by themselves.  So consecutive calls may overlap when the caller allows it.
+// partials, the only workspace data that the next call overwrites.  (A call of this
+// kernel clears the tickets first; pipelined calls run k_tiles + k_finish instead.)
 template <typename T, bool VEC, int VPT, bool VEC4, int RESID, int RU>
 __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs A) {
   __shared__ float2 red[kK1Threads / 32];
@@ -792,7 +804,7 @@ __global__ void __launch_bounds__(kK1Threads, kK1MinBlocks) k_verify(VerifyArgs 
 // With many chains the fused kernel's finishing CTAs (each holding a CTA slot for
 // the whole latency-bound scan / U-draw / residual) take more SM time than the
 // stream itself.  The many-chain path streams the same tiles without tickets
-// (k_tiles: identical partials) at full occupancy, then finishes every chain with
+// (k_tiles: identical partials, tagged with the call) at full occupancy, then finishes every chain with
 // a small CTA (k_finish: one warp's scan and U-draw, then the residual row), all
 // chains at once.
 // One tile's 3 VPT 16-byte vectors per thread (a tile is one full sweep: VPT vectors
@@ -853,9 +865,8 @@ __device__ __forceinline__ float2 tile_fma(const TileBuf<VPT>& B) {
 }
 
 // The stream of the many-chain and pipelined paths: one tile per CTA; its (S1, S2) is
-// stored and counted on its chain (red.release.inc, wrapping to 0 at the chain's last
-// tile).  The FMAs of a tile and their order are those of tile_sums, so the partials
-// equal the fused kernel's.  (Two or four software-pipelined tiles per CTA measured
+// stored with the call's tag.  The FMAs of a tile and their order are those of
+// tile_sums, so the partials equal the fused kernel's.  (Two or four software-pipelined tiles per CTA measured
 // slower: 17.4 / 20.1 us against 16.5 us per pipelined pixel call.)
 template <typename T, bool VEC, int VPT>
 __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(VerifyArgs A) {
@@ -880,10 +891,12 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
     }
     const float2 t = block_sum2<kK1Threads>(sm.x, sm.y, red);
     if (threadIdx.x == 0) {
-      A.part[tile] = t;
-      // release the partial with the chain's count, which wraps to 0 at the chain's
-      // last tile; k_finish acquires every partial of the chain by reading that 0
-      ticket_inc_noret(A.ticket + b, (unsigned int)(g * C) - 1u);
+      // S1 and S2 each share an 8-byte word with the call's tag; each word is written
+      // whole (a vector of two 8-byte elements), so k_finish can tell this call's
+      // partials from those a previous call left in the slot
+      const unsigned long long tg = (unsigned long long)A.S.tag << 32;
+      reinterpret_cast<ulonglong2*>(A.tpart)[tile] =
+          make_ulonglong2(tg | __float_as_uint(t.x), tg | __float_as_uint(t.y));
     }
   }
   if (blockIdx.x == 0) {
@@ -896,9 +909,10 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   }
 }
 
-// One CTA per chain: warp 0 reads the chain's partials (after acquiring its tile count,
-// complete -- and wrapped back to 0 -- because k_finish starts only after every k_tiles
-// CTA has taken its ticket and exited or triggered), and the CTA triggers its dependents; then warp 0 scans the chain and draws U
+// One CTA per chain: warp 0 reads the chain's partials (k_finish starts only after
+// every k_tiles CTA has stored its partial and exited or triggered; the tags confirm
+// that each one read is this call's, else the warp waits for k_tiles to complete and
+// reads them again), and the CTA triggers its dependents; then warp 0 scans the chain and draws U
 // (warp U-sampler) while the other warps draw the residual's G into shared memory
 // (dynamic, (d + 3)/4 float4), and, with RESID = 1, all kFinishThreads threads write y
 // (launched with 32 threads and leaving the chain state for k_resid_* when RESID = 0).
@@ -918,15 +932,15 @@ __global__ void __launch_bounds__(NT) k_finish(VerifyArgs A) {
   const int L = A.S.L;
   ScanRegs R;
   if (threadIdx.x < 32) {
-    if (threadIdx.x == 0) {
-      // the count is back at 0 after the chain's last tile: reading it with acquire
-      // semantics makes every partial released by the chain's tiles visible
-      uint32_t cnt;
-      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(cnt) : "l"(A.ticket + b) : "memory");
-      (void)cnt;
-    }
-    __syncwarp();
     R = scan_load(A.S, b);
+    if (R.stale) {
+      // a partial of this call is not visible yet (k_finish starts once every k_tiles
+      // CTA has stored its partial and exited or triggered, so in practice they all
+      // are): wait for k_tiles to complete, which makes its writes visible, and read
+      // them again
+      griddep_wait();
+      R = scan_load(A.S, b, false);
+    }
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
       if (threadIdx.x + 32 * q < L) {
@@ -1182,10 +1196,14 @@ static void timing_record(cudaEvent_t e, cudaStream_t s) {
 WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   WsLayout w{};
   const int es = dtype == SDV_BF16 ? 2 : 4;
-  // vectors per thread: the smallest sweep that covers a row, capped at kK1Vpt,
-  // so that common row lengths run whole, unguarded sweeps
+  // vectors per thread: the smallest sweep that covers a row, capped at kK1Vpt (at 2
+  // for bf16 rows, whose 16-byte vectors hold 8 elements: the 40-register tiles leave
+  // room on an SM for the previous pipelined call's 256-thread finishing CTA; latent
+  // rows 19.5 -> 19.0 us per pipelined call), so that common row lengths run whole,
+  // unguarded sweeps
   const int64_t vec_per_row = (d * es + 15) / 16;
-  w.vpt1 = (int)std::min<int64_t>(kK1Vpt, std::max<int64_t>(1, (vec_per_row + kK1Threads - 1) / kK1Threads));
+  const int64_t vpt_cap = es == 2 ? 2 : kK1Vpt;
+  w.vpt1 = (int)std::min<int64_t>(vpt_cap, std::max<int64_t>(1, (vec_per_row + kK1Threads - 1) / kK1Threads));
   w.chunk1 = (int64_t)kK1Threads * w.vpt1 * (16 / es);
   w.C1 = (int)((d + w.chunk1 - 1) / w.chunk1);
   // long-row residual chunks: about kK4TargetCtas CTAs over all chains, kK4MinChunk ..
@@ -1199,7 +1217,7 @@ WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   w.ticket_off = off;
   off = up(off + sizeof(unsigned int) * (size_t)B);
   w.part_off = off;
-  off = up(off + sizeof(float2) * (size_t)B * L * w.C1);
+  off = up(off + 2 * sizeof(uint64_t) * (size_t)B * L * w.C1);
   w.state_off = off;
   off = up(off + sizeof(ChainState) * (size_t)B);
   w.part4_off = off;
@@ -1366,6 +1384,19 @@ static cudaError_t launch_k4(const void* x, const void* mq, const void* mp, cons
   return e;
 }
 
+// The tag of a call's k_tiles partials: a process-wide counter, never 0 (a zeroed
+// workspace holds tag 0), so consecutive calls on a workspace never share a tag (a
+// captured call keeps its tag at every replay of its graph, and replays of a graph run
+// one after another).
+static std::atomic<uint32_t> g_partial_tag{0u};
+static uint32_t next_partial_tag() {
+  uint32_t t;
+  do {
+    t = g_partial_tag.fetch_add(1u, std::memory_order_relaxed) + 1u;
+  } while (t == 0u);
+  return t;
+}
+
 // Enqueue the whole step (or, with ratios_only, the log-ratio pass) for validated args.
 static int enqueue_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
                           const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d,
@@ -1385,7 +1416,9 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   A.state = (ChainState*)(ws + w.state_off);
   ScanArgs& S = A.S;
   A.part = (float2*)(ws + w.part_off);
-  S.part = A.part; S.C = w.C1; S.sigma = sigma; S.sstride = sigma_stride_b;
+  A.tpart = (uint64_t*)(ws + w.part_off);
+  S.part = A.part; S.tpart = nullptr; S.tag = 0u;
+  S.C = w.C1; S.sigma = sigma; S.sstride = sigma_stride_b;
   S.B = B; S.L = L; S.L_eff = L_eff; S.seed = seed; S.seed_dev = seed_dev; S.mode = mode;
   S.inv_omega2 = 1.0f / (omega * omega); S.residual_kind = residual_kind;
   S.has_bonus = mu_target_bonus != nullptr; S.ratios_only = ratios_only; S.draw_u = true;
@@ -1409,9 +1442,13 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   const bool long_rows = !ratios_only && !wide && ng > (many ? kFinishMaxGroups : kFusedMaxGroups);
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;
-  // the tickets return to zero at the end of every call; a pipelined call relies on
-  // that (the caller's contract), the others clear them first
-  if (!overlap && cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+  if (many) {
+    // k_tiles + k_finish: tagged partials, no counters
+    S.part = nullptr;
+    S.tpart = A.tpart;
+    S.tag = next_partial_tag();
+  } else if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
+    // the fused kernel counts the tiles of each chain from zero
     check_launch();
     return SDV_ECUDA;
   }
@@ -1434,8 +1471,8 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   if (rc != SDV_OK) return rc;
   if (tev) timing_record(tev[1], s);
   // The kernels after the first of a call are always launched to overlap their
-  // predecessor within the call: k_finish reads nothing before every k_tiles CTA has
-  // counted its tile, and the residual kernels wait for their inputs at their start;
+  // predecessor within the call: k_finish starts once every k_tiles CTA has stored
+  // its partial (and checks their tags), and the residual kernels wait for their inputs at their start;
   // only the first kernel's overlap with the previous call needs the pipelined contract.
   if (many) {
     if (long_rows)

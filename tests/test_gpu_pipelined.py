@@ -7,7 +7,8 @@ every chain with k_finish (the one-warp U-sampler, a 64-thread residual writer),
 U and states agree with a plain call's within the parity tolerances (U: 5e-6 + 3e-7|U|;
 states: 1e-5 absolute for fp32, 2e-2 for bf16), and one run is compared with the oracle
 directly.  Checked with separate outputs per call, with outputs shared by all calls
-(written in call order), and under CUDA-graph capture."""
+(written in call order), under CUDA-graph capture, and with one workspace of arbitrary
+contents reused by calls of changing sizes."""
 import numpy as np
 import pytest
 import torch
@@ -177,3 +178,20 @@ def test_pipelined_long_rows_many_chains(api):
     torch.cuda.synchronize()
     for i in range(2):
         _same(piped[i], _call(api, sets[0], 700 + i, "sample", ws))
+
+
+def test_pipelined_calls_reuse_a_workspace_across_sizes(api):
+    """One workspace of arbitrary contents (filled with 0xFF bytes) serves a run of
+    pipelined calls whose sizes change from call to call, so that each call's tile
+    partials land on slots that a call of other sizes left behind: the partials' tags
+    keep every call to its own (against plain calls on a fresh workspace)."""
+    shapes = [(64, 8, 3072), (160, 4, 1000), (96, 8, 3072), (72, 6, 2048), (200, 2, 520)]
+    sets = {sh: _sets("pixel", 1, *sh, False)[0] for sh in shapes}
+    nbytes = max(api.workspace_bytes(B, L, d, torch.float32) for B, L, d in shapes)
+    ws = torch.full((nbytes,), 255, dtype=torch.uint8, device="cuda")
+    order = shapes + shapes[::-1] + shapes
+    piped = [_call(api, sets[sh], 900 + i, "block", ws, pipelined=True) for i, sh in enumerate(order)]
+    torch.cuda.synchronize()
+    for i, sh in enumerate(order):
+        fresh = torch.zeros(api.workspace_bytes(*sh, torch.float32), dtype=torch.uint8, device="cuda")
+        _same(piped[i], _call(api, sets[sh], 900 + i, "block", fresh))

@@ -82,7 +82,9 @@ struct ChainState {
 struct ScanArgs {
   const float2* part;     // fused kernel: [B, L, C] (S1, S2) per tile
   const uint64_t* tpart;  // k_tiles: [B, L, C] pairs of words (S1 | tag << 32, S2 | tag << 32)
+  uint32_t* consumed;     // [B, L, C] beside tpart: the tag of the partial last read from each slot
   uint32_t tag;           // this call's tag of its k_tiles partials (never 0)
+  bool fresh_set;         // the set held another layout before: k_tiles waits before its stores
   int C;
   const float* sigma;
   int64_t sstride;
@@ -113,9 +115,10 @@ struct WsLayout {
   int C1;          // K1 tiles per row
   int64_t chunk4;  // K4 elements per tile
   int C4;          // K4 tiles per chain
-  // tickets [B] u32 (fused kernel), tile partials [B, L, C1] 16 bytes each (the fused
-  // kernel's float2 or k_tiles' tagged pair of words), chain states, long-row partials
-  size_t ticket_off, part_off, state_off, part4_off, total;
+  // tickets [B] u32 (fused kernel); two sets of tile partials [B, L, C1], 16 bytes
+  // each (the fused kernel's float2, in set 0, or k_tiles' tagged pair of words), each
+  // followed by its consumed tags [B, L, C1] u32; chain states; long-row partials
+  size_t ticket_off, part_off, part_set_bytes, cons_off, state_off, part4_off, total;
 };
 
 WsLayout ws_layout(int B, int L, int64_t d, int dtype);

@@ -23,6 +23,7 @@
 
 #include <algorithm>
 #include <atomic>
+#include <mutex>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -246,7 +247,8 @@ __device__ ScanRegs scan_load(const ScanArgs& A, int b, bool check_tags = true) 
         // in tile order
         float a1 = 0.f, a2 = 0.f;
         if (A.tpart) {
-          const ulonglong2* p = reinterpret_cast<const ulonglong2*>(A.tpart) + ((int64_t)b * L + j) * A.C;
+          const int64_t s0 = ((int64_t)b * L + j) * A.C;
+          const ulonglong2* p = reinterpret_cast<const ulonglong2*>(A.tpart) + s0;
 #pragma unroll 4
           for (int c = 0; c < A.C; ++c) {
             const ulonglong2 t = __ldcg(p + c);
@@ -864,6 +866,14 @@ __device__ __forceinline__ float2 tile_fma(const TileBuf<VPT>& B) {
   return make_float2(s1, s2);
 }
 
+// The tag of the partial in slot `tile` of this call's set and the tag its reader
+// released after reading it (acquire: the reader's loads of the slot happen before
+// anything this thread does next).
+__device__ __forceinline__ void slot_state(const VerifyArgs& A, int64_t tile, uint32_t& held, uint32_t& taken) {
+  held = __ldcg(reinterpret_cast<const unsigned int*>(A.tpart + 2 * tile) + 1);
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(taken) : "l"(A.S.consumed + tile) : "memory");
+}
+
 // The stream of the many-chain and pipelined paths: one tile per CTA; its (S1, S2) is
 // stored with the call's tag.  The FMAs of a tile and their order are those of
 // tile_sums, so the partials equal the fused kernel's.  (Two or four software-pipelined tiles per CTA measured
@@ -881,16 +891,27 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   if (j < g) {  // CTA-uniform
     const int64_t e0 = (int64_t)c * A.chunk;
     const int64_t e1 = min(e0 + A.chunk, A.d);
+    // the tag now in this CTA's slot and the tag last consumed from it, loaded by thread
+    // 0 once its tile loads are in flight (the acquire orders only what follows it) and
+    // compared before the store
+    uint32_t held = 0u, taken = 0u;
     float2 sm;
     if (VEC) {
       TileBuf<VPT> B;
       tile_issue<T, VPT>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1, B);
+      if (threadIdx.x == 0) slot_state(A, tile, held, taken);
       sm = tile_fma<T, VPT>(B);
     } else {
+      if (threadIdx.x == 0) slot_state(A, tile, held, taken);
       sm = tile_sums<T, false, 1>((const T*)A.x, (const T*)A.mq, (const T*)A.mp, r * A.d, e0, e1);
     }
     const float2 t = block_sum2<kK1Threads>(sm.x, sm.y, red);
     if (threadIdx.x == 0) {
+      // the slot's partial has not been read yet by the call that wrote it (which may
+      // still be finishing, since calls overlap), or this set held another layout:
+      // wait for the previous kernel, whose completion implies every earlier call's
+      // (in practice the slot was read long ago)
+      if (A.S.fresh_set || held != taken) griddep_wait();
       // S1 and S2 each share an 8-byte word with the call's tag; each word is written
       // whole (a vector of two 8-byte elements), so k_finish can tell this call's
       // partials from those a previous call left in the slot
@@ -926,11 +947,15 @@ __global__ void __launch_bounds__(NT) k_finish(VerifyArgs A) {
   __shared__ UParams P_s;
   __shared__ bool haveP_s;
   __shared__ USampleScratch us;
+  __shared__ int gw_s;             // the chain's window length (tiles written this call)
   extern __shared__ float4 g_s[];  // RESID: the residual's G, drawn once
   constexpr int RU = NT >= 256 ? kFusedResidUnroll : kFinishResidUnroll;
   const int b = blockIdx.x;
   const int L = A.S.L;
   ScanRegs R;
+  // the next kernel (the next call's stream) may start now: it writes the other set of
+  // partials, and a slot of this set only once this call has read it
+  griddep_launch_dependents();
   if (threadIdx.x < 32) {
     R = scan_load(A.S, b);
     if (R.stale) {
@@ -948,9 +973,19 @@ __global__ void __launch_bounds__(NT) k_finish(VerifyArgs A) {
         dn_s[threadIdx.x + 32 * q] = R.dn[q];
       }
     }
+    if (threadIdx.x == 0) gw_s = R.g;
   }
   __syncthreads();
-  griddep_launch_dependents();  // this chain's partials are read
+  if (A.S.consumed && (int)(threadIdx.x >> 5) == (NT > 32 ? 1 : 0)) {
+    // release the chain's slots (those its tiles wrote) to the next call that writes
+    // this set: the barrier orders warp 0's reads of them before these stores, and that
+    // call's k_tiles CTA overwrites a slot once it reads back (acquire) the tag it found
+    // there.  Off warp 0's path where the CTA has a second warp.
+    const int64_t s0 = (int64_t)b * L * A.S.C;
+    const int n = gw_s * A.S.C;
+    for (int k = threadIdx.x & 31; k < n; k += 32)
+      asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(A.S.consumed + s0 + k), "r"(A.S.tag) : "memory");
+  }
   if (threadIdx.x < 32) {
     const ScanOut so = scan_decide(A.S, b, R);
     ChainState cs = so.cs;
@@ -1217,7 +1252,10 @@ WsLayout ws_layout(int B, int L, int64_t d, int dtype) {
   w.ticket_off = off;
   off = up(off + sizeof(unsigned int) * (size_t)B);
   w.part_off = off;
-  off = up(off + 2 * sizeof(uint64_t) * (size_t)B * L * w.C1);
+  const size_t slots = (size_t)B * L * w.C1;
+  w.cons_off = up(2 * sizeof(uint64_t) * slots);  // within a set
+  w.part_set_bytes = up(w.cons_off + sizeof(uint32_t) * slots);
+  off = up(off + 2 * w.part_set_bytes);
   w.state_off = off;
   off = up(off + sizeof(ChainState) * (size_t)B);
   w.part4_off = off;
@@ -1397,6 +1435,32 @@ static uint32_t next_partial_tag() {
   return t;
 }
 
+// The set of partials a call on `workspace` uses: the other one than the previous call
+// on that workspace (remembered for the last kPartialSetSlots workspaces; a forgotten
+// workspace starts again at set 0, which at worst makes a stream CTA wait for the
+// previous kernel before its store).
+// `fresh` when the set's last user on this workspace had another layout (or is
+// unknown): the stream then waits for the previous kernel before it stores.
+constexpr int kPartialSetSlots = 64;
+static int next_partial_set(const void* workspace, uint64_t layout, bool* fresh) {
+  struct Entry {
+    const void* ws;
+    int next;
+    uint64_t layout[2];
+  };
+  static std::mutex mu;
+  static Entry tab[kPartialSetSlots] = {};
+  const size_t h = (reinterpret_cast<uintptr_t>(workspace) >> 8) % kPartialSetSlots;
+  std::lock_guard<std::mutex> lock(mu);
+  Entry& e = tab[h];
+  if (e.ws != workspace) e = Entry{workspace, 0, {0u, 0u}};
+  const int set = e.next;
+  *fresh = e.layout[set] != layout;
+  e.layout[set] = layout;
+  e.next ^= 1;
+  return set;
+}
+
 // Enqueue the whole step (or, with ratios_only, the log-ratio pass) for validated args.
 static int enqueue_verify(const void* x_draft, const void* mu_target, const void* mu_draft,
                           const float* sigma, int64_t sigma_stride_b, int B, int L, int64_t d,
@@ -1417,7 +1481,7 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   ScanArgs& S = A.S;
   A.part = (float2*)(ws + w.part_off);
   A.tpart = (uint64_t*)(ws + w.part_off);
-  S.part = A.part; S.tpart = nullptr; S.tag = 0u;
+  S.part = A.part; S.tpart = nullptr; S.consumed = nullptr; S.tag = 0u; S.fresh_set = false;
   S.C = w.C1; S.sigma = sigma; S.sstride = sigma_stride_b;
   S.B = B; S.L = L; S.L_eff = L_eff; S.seed = seed; S.seed_dev = seed_dev; S.mode = mode;
   S.inv_omega2 = 1.0f / (omega * omega); S.residual_kind = residual_kind;
@@ -1443,9 +1507,17 @@ static int enqueue_verify(const void* x_draft, const void* mu_target, const void
   const bool f32 = dtype == SDV_F32;
   cudaError_t e = cudaSuccess;
   if (many) {
-    // k_tiles + k_finish: tagged partials, no counters
+    // k_tiles + k_finish: tagged partials in the set after the one this workspace's
+    // previous call used, no counters
+    // the layout key: the slot count and the set's size (never 0)
+    const uint64_t layout = ((uint64_t)B * L * w.C1 << 24) ^ (uint64_t)w.part_set_bytes ^ 1u;
+    bool fresh = true;
+    char* set = ws + w.part_off + (size_t)next_partial_set(workspace, layout, &fresh) * w.part_set_bytes;
+    S.fresh_set = fresh;
+    A.tpart = (uint64_t*)set;
     S.part = nullptr;
     S.tpart = A.tpart;
+    S.consumed = (uint32_t*)(set + w.cons_off);
     S.tag = next_partial_tag();
   } else if (cudaMemsetAsync(A.ticket, 0, sizeof(unsigned int) * (size_t)B, s) != cudaSuccess) {
     // the fused kernel counts the tiles of each chain from zero

@@ -930,10 +930,12 @@ __global__ void __launch_bounds__(kK1Threads, tile_min_blocks(VPT)) k_tiles(Veri
   }
 }
 
-// One CTA per chain: warp 0 reads the chain's partials (k_finish starts only after
-// every k_tiles CTA has stored its partial and exited or triggered; the tags confirm
-// that each one read is this call's, else the warp waits for k_tiles to complete and
-// reads them again), and the CTA triggers its dependents; then warp 0 scans the chain and draws U
+// One CTA per chain: the CTA triggers its dependents at once (the next call's stream
+// writes the other set of partials); warp 0 reads the chain's partials (k_finish starts
+// only after every k_tiles CTA has stored its partial and exited or triggered; the tags
+// confirm that each one read is this call's, else the warp waits for k_tiles to
+// complete and reads them again), and after the barrier a second warp releases the
+// chain's slots to the next call that writes this set; then warp 0 scans the chain and draws U
 // (warp U-sampler) while the other warps draw the residual's G into shared memory
 // (dynamic, (d + 3)/4 float4), and, with RESID = 1, all kFinishThreads threads write y
 // (launched with 32 threads and leaving the chain state for k_resid_* when RESID = 0).

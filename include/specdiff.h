@@ -165,9 +165,11 @@ int sdv_verify_ex(const void *x_draft, const void *mu_target, const void *mu_dra
  * mu_target, mu_draft, sigma, L_eff, mu_target_bonus, sigma_bonus) is not written by
  * earlier work on `stream` that may still be running: the previous kernel, and the
  * earlier calls of a run of pipelined calls (the window is read while they finish).
- * The workspace needs no preparation: each tile partial is stored with a tag of its
- * call, and the finishing kernel waits for the whole stream of its call when it reads
- * a partial without that tag.
+ * The workspace needs no preparation: its two sets of tile partials are used
+ * alternately by consecutive calls, each partial stored with a tag of its call; a
+ * stream overwrites a slot only after the call that wrote it has read it (else it
+ * waits for the previous kernel), and the finishing kernel waits for the whole stream
+ * of its call when it reads a partial without its call's tag.
  * Outputs are written only after the previous call on `stream` has written its own,
  * so consecutive calls may share output buffers.  Rows longer than 16384 elements
  * add two residual kernels, which overlap the next call's stream too.  Same
